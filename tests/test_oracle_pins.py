@@ -1,0 +1,113 @@
+"""The fp64 oracle against what the paper and mathematics fix (CPU only)."""
+import numpy as np
+import pytest
+
+import oracle
+import pins
+
+
+@pytest.mark.parametrize("name,case", pins.golden_cases(), ids=[n for n, _ in pins.golden_cases()])
+def test_golden(orc, name, case):
+    pins.check_golden(orc, case)
+
+
+@pytest.mark.parametrize("n,d", [(2, 1), (5, 3), (64, 16), (300, 64)])
+def test_decomp_identity(orc, n, d):
+    pins.check_decomp(orc, pins.gauss_cache(np.random.default_rng(n * d), n, d))
+
+
+@pytest.mark.parametrize("n,d", [(2, 3), (3, 1), (9, 4), (12, 8)])
+def test_uniform_attention_reconstruction(orc, n, d):
+    pins.check_recon_error(orc, pins.gauss_cache(np.random.default_rng(n + d), n, d))
+
+
+@pytest.mark.parametrize("n,d", [(3, 2), (8, 6)])
+def test_dirichlet_identities(orc, n, d):
+    pins.check_dirichlet_identities(orc, pins.gauss_cache(np.random.default_rng(7 * n), n, d))
+
+
+@pytest.mark.parametrize("n", [3, 5, 8])
+def test_dirichlet_expectation_monte_carlo(orc, n):
+    rng = np.random.default_rng(100 + n)
+    pins.check_dirichlet_mc(orc, pins.gauss_cache(rng, n, 4, outliers=False), rng)
+
+
+def test_distance_from_symmetric_limit(orc):
+    rng = np.random.default_rng(5)
+    for n in (4, 6, 9):
+        pins.check_distance_bound(orc, pins.gauss_cache(rng, n, 5), rng)
+
+
+@pytest.mark.parametrize("shift", [1.0, -7.0, 32.0])
+def test_translation_invariance(orc, shift):
+    pins.check_translation(orc, pins.int_cache(np.random.default_rng(3), 50, 8), shift)
+
+
+@pytest.mark.parametrize("power", [-4, 1, 6])
+def test_positive_homogeneity(orc, power):
+    pins.check_homogeneity(orc, pins.gauss_cache(np.random.default_rng(4), 64, 16), power, 20)
+
+
+def test_permutation_equivariance(orc):
+    rng = np.random.default_rng(6)
+    for n in (10, 47):
+        pins.check_permutation(orc, pins.gauss_cache(rng, n, 8), rng.permutation(n), n // 3)
+
+
+@pytest.mark.parametrize("seed", range(6))
+def test_top_n_brute_force(orc, seed):
+    rng = np.random.default_rng(seed)
+    n = int(rng.integers(1, 60))
+    s = rng.integers(0, 5, size=n).astype(np.float64) if seed % 2 else rng.normal(size=n)
+    for N in sorted({1, max(1, n // 2), max(1, n - 1), n, n + 3}):
+        pins.check_top_n(orc, s, N)
+
+
+@pytest.mark.parametrize("var", [oracle.L2, oracle.DIR, oracle.NORM])
+def test_gather_matches_out_of_place(orc, var):
+    rng = np.random.default_rng(8)
+    for n, N in ((1, 1), (20, 19), (33, 5), (64, 64), (80, 100)):
+        pins.check_gather(orc, rng, n, 8, N, var)
+
+
+def test_special_cases(orc):
+    pins.check_special_cases(orc, np.random.default_rng(9))
+
+
+def test_block_equivalences(orc):
+    pins.check_block_equivalences(orc, np.random.default_rng(10))
+
+
+def test_batched_units_match_single_units(orc):
+    """The threaded many-unit entry point (the CPU baseline) is the per-unit
+    eviction applied to each unit with that unit's sequence length and budget."""
+    rng = np.random.default_rng(11)
+    n_seq, per_seq, cap, d = 3, 4, 40, 8
+    U = n_seq * per_seq
+    k = np.stack([pins.gauss_cache(rng, cap, d) for _ in range(U)])
+    v = np.stack([pins.gauss_cache(rng, cap, d) for _ in range(U)])
+    lens = np.array([40, 17, 30], np.int32)
+    Ns = np.array([25, 20, 29], np.int32)
+    k1, v1 = k.copy(), v.copy()
+    kept = orc.evict_units(k1, v1, lens, Ns, per_seq, oracle.DIR, nthreads=4, kept_stride=29)
+    for u in range(U):
+        s = u // per_seq
+        n = lens[s]
+        k2, v2, kp, _ = orc.evict_unit(k[u, :n], v[u, :n], int(Ns[s]), oracle.DIR)
+        m = len(kp)
+        assert np.array_equal(kept[u, :m], kp) and np.all(kept[u, m:] == -1)
+        assert np.array_equal(v1[u, :m], v2) and np.array_equal(k1[u, :m], k2)
+        assert np.array_equal(v1[u, m:], v[u, m:])   # slots past the new length untouched
+
+
+def test_sum_rows_is_exact_for_bf16(orc):
+    """fp64 sums of bf16 rows of moderate range are exact: the compensated sum
+    equals an exact rational sum."""
+    from fractions import Fraction
+    rng = np.random.default_rng(12)
+    v = pins.gauss_cache(rng, 500, 4)
+    x = pins.as_float(v)
+    got = orc.sum_rows(v)
+    for c in range(4):
+        exact = sum(Fraction(float(t)) for t in x[:, c])
+        assert got[c] == float(exact)
