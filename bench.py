@@ -1,0 +1,651 @@
+"""Benchmark of the ValueDiff eviction hot path on GB300.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl vd|reference]
+                    [--workload prefill_wide|decode_batched|prefill_gqa8b|ratio_budget|tiny_prefill]
+
+One step = one eviction event of the whole hot path over every unit of the
+workload: the block (or token) append of Eq. (block_processing) followed by
+pi_N (mean -> scores -> top-N -> in-place K/V compaction).  The workload is
+at steady state (cache at N before each append), inputs are resident in HBM
+and larger than L2.  Prints one JSON line (rank 0):
+
+  value       head-tokens scored and compacted per second, whole job
+  roofline    the fused eviction kernel: algorithmic bytes per launch / its
+              CUDA-event duration, against the measured HBM copy bandwidth
+  e2e         the same metric through the C ABI with the step's new K/V rows
+              copied from pinned host memory and the step's result (kept or
+              evicted slots) copied back, every step
+  cpu_baseline  the fp64 CPU oracle on a bounded sample of the same events
+  secondary   the largest decode workload measured the same way (default run)
+
+--impl reference times the oracle itself (the CPU reference of this build).
+Multi-GPU (torchrun): every rank runs its own replica of the workload (units
+are independent; no collective on the data path) -> weak scaling; the step
+time is the max over ranks.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "cache tokens scored+compacted/s; HBM GB/s as % of GB300 peak per eviction"
+UNIT = "head-tokens/s"
+FALLBACK_HBM_GBS = 6800.0
+L2_BYTES = 129 * 2 ** 20
+
+
+# ---------------------------------------------------------------------------
+# host logic shared by all ranks (tested on CPU with gloo)
+# ---------------------------------------------------------------------------
+def dist_env():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", str(rank)))
+    return ws, rank, local
+
+
+def rank_seed(base: int, rank: int) -> int:
+    """Each rank's replica draws its own inputs."""
+    return base + 1000 * rank
+
+
+def max_over_ranks(value: float, device=None) -> float:
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()):
+        return value
+    t = torch.tensor([value], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def barrier(device=None):
+    import torch.distributed as dist
+    if dist.is_available() and dist.is_initialized():
+        if device is not None and str(device).startswith("cuda"):
+            dist.barrier(device_ids=[device.index if hasattr(device, "index") else 0])
+        else:
+            dist.barrier()
+
+
+def whole_job_rate(units_per_rank_step: float, steps: int, world: int, max_ms: float) -> float:
+    return units_per_rank_step * steps * world / (max_ms / 1e3)
+
+
+# ---------------------------------------------------------------------------
+# measured peaks, clocks, ncu traffic
+# ---------------------------------------------------------------------------
+def hbm_peak():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return float(p["hbm_gbs"]), "measured (MEASURED_PEAKS.json hbm_gbs)"
+    except Exception:
+        return FALLBACK_HBM_GBS, "fallback (no MEASURED_PEAKS.json)"
+
+
+def kernel_source_hash() -> str:
+    h = hashlib.sha256()
+    csrc = os.path.join(ROOT, "paper_2609_23314_gb300", "csrc")
+    for name in sorted(os.listdir(csrc)):
+        with open(os.path.join(csrc, name), "rb") as f:
+            h.update(name.encode() + f.read())
+    return h.hexdigest()[:16]
+
+
+def ncu_traffic(workload: str):
+    """DRAM bytes per launch of the eviction kernel from the committed ncu
+    summary, if it was taken on the current kernel sources; else None."""
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    try:
+        with open(path) as f:
+            t = json.load(f)
+        e = t[workload]
+        if e.get("source_hash") != kernel_source_hash():
+            return None
+        return float(e["dram_bytes_per_launch"])
+    except Exception:
+        return None
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons sampled during the timed region."""
+
+    FIELDS = ("clocks.sm,clocks.max.sm,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.lines = []
+        self._t = None
+        self.window = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "50"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self._t = threading.Thread(target=self._read, daemon=True)
+            self._t.start()
+        except Exception:
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append((time.time(), line.strip()))
+
+    def mark(self, t0, t1):
+        self.window = (t0, t1)
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        if self._t:
+            self._t.join(timeout=2)
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        lines = self.lines
+        if self.window is not None:
+            inside = [ln for ts, ln in lines if self.window[0] <= ts <= self.window[1] + 0.06]
+            lines = inside if inside else [ln for _, ln in lines[-3:]]
+        else:
+            lines = [ln for _, ln in lines]
+        for ln in lines:
+            parts = [p.strip() for p in ln.split(",")]
+            if len(parts) < 7:
+                continue
+            try:
+                sm.append(float(parts[0]))
+                mx.append(float(parts[1]))
+            except ValueError:
+                continue
+            for nm, val in zip(names, parts[3:7]):
+                if val.lower() == "active":
+                    reasons.add(nm)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"], "samples": 0}
+        sm.sort()
+        return {"sm_mhz": sm[len(sm) // 2], "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# ---------------------------------------------------------------------------
+# workloads at steady state
+# ---------------------------------------------------------------------------
+class Prefill:
+    """Block boundary at steady state: append B rows, evict N + B -> N."""
+
+    def __init__(self, name, cfg, device, seed, mu, variant, n_blocks=8):
+        import torch
+        import paper_2609_23314_gb300 as vd
+        from paper_2609_23314_gb300 import workloads as wl
+        self.vd, self.torch = vd, torch
+        self.name, self.cfg, self.device = name, cfg, device
+        self.N, self.B, self.d = cfg["N"], cfg["B"], cfg["head_dim"]
+        self.cap = self.N + self.B
+        self.cache = vd.Cache.empty(cfg["n_seq"], cfg["n_layer"], cfg["n_kv_head"], self.cap,
+                                    self.d, device=device)
+        self.U = self.cache.units
+        st = wl.stream_for(cfg, device=str(device), seed=seed)
+        kv = self.cache.k.view(self.U, self.cap, self.d), self.cache.v.view(self.U, self.cap, self.d)
+        wl.fill_rows(st, kv[0], kv[1], self.N, chunk_units=64)
+        self.cache.len.fill_(self.N)
+        us = self.cache.unit_shape()
+        self.blocks = []
+        for _ in range(n_blocks):
+            k, v = st.next(self.B)
+            self.blocks.append((k.view(us + (self.B, self.d)).contiguous(),
+                                v.view(us + (self.B, self.d)).contiguous()))
+        self.mu, self.variant = mu, variant
+        self.rs = torch.zeros(us + (self.d,), dtype=torch.float64, device=device)
+        if mu == vd.VD_MU_RUNNING:
+            vd.vd_running_sum_init(self.cache, self.rs)
+        self.kept = None
+        self.i = 0
+        self.launches_per_step = 4     # append + len add, evict + len clamp
+
+    def head_tokens_per_step(self):
+        return self.U * (self.N + self.B)
+
+    def new_kept_buffers(self, k):
+        t = self.torch
+        return [t.empty(self.cache.unit_shape() + (self.N,), dtype=t.int32, device=self.device)
+                for _ in range(k)]
+
+    def step(self, kept=None, ev=None):
+        vd = self.vd
+        k, v = self.blocks[self.i % len(self.blocks)]
+        self.i += 1
+        vd.vd_append(self.cache, k, v, self.B)
+        if ev is not None:
+            ev[0].record()
+        vd.vd_evict_block(self.cache, self.N, None, self.B, self.variant, self.mu,
+                          self.rs if self.mu else None, kept, None)
+        if ev is not None:
+            ev[1].record()
+
+    def moved_rows(self, kept_list):
+        """Rows of one unit moved by the compaction: N - first evicted slot."""
+        t = self.torch
+        total = 0
+        ar = t.arange(self.N, device=self.device, dtype=t.int32)
+        for kp in kept_list:
+            kk = kp.view(self.U, self.N)
+            same = (kk == ar)
+            first = t.where(same.all(dim=1), t.full((self.U,), self.N, device=self.device),
+                            (~same).int().argmax(dim=1))
+            total += int((self.N - first).sum().item())
+        return total / max(1, len(kept_list))
+
+    def bytes_per_launch(self, moved_rows_total):
+        n, d = self.N + self.B, self.d
+        v_read = self.U * n * d * 2
+        move = moved_rows_total * d * 2 * 2 * 2
+        extra = self.U * d * 8 * 2 if self.mu else 0
+        return v_read + move + extra, v_read + self.U * self.N * d * 2 * 2 * 2 + extra
+
+    # e2e through the C ABI with host buffers
+    def e2e_setup(self):
+        t = self.torch
+        us = self.cache.unit_shape()
+        self.h_blocks = [(k.cpu().pin_memory(), v.cpu().pin_memory()) for k, v in self.blocks[:2]]
+        self.d_k = t.empty(us + (self.B, self.d), dtype=t.bfloat16, device=self.device)
+        self.d_v = t.empty_like(self.d_k)
+        self.d_kept = t.empty(us + (self.N,), dtype=t.int32, device=self.device)
+        self.h_kept = t.empty(us + (self.N,), dtype=t.int32).pin_memory()
+        bi = 2 * self.d_k.numel() * 2
+        bo = self.d_kept.numel() * 4
+        return bi, bo
+
+    def e2e_step(self):
+        vd = self.vd
+        hk, hv = self.h_blocks[self.i % 2]
+        self.i += 1
+        self.d_k.copy_(hk, non_blocking=True)
+        self.d_v.copy_(hv, non_blocking=True)
+        vd.vd_append(self.cache, self.d_k, self.d_v, self.B)
+        vd.vd_evict_block(self.cache, self.N, None, self.B, self.variant, self.mu,
+                          self.rs if self.mu else None, self.d_kept, None)
+        self.h_kept.copy_(self.d_kept, non_blocking=True)
+
+    # oracle sample: the pre-eviction bytes of a few units at steady state
+    def oracle_sample(self, units):
+        t = self.torch
+        vd = self.vd
+        k, v = self.blocks[0]
+        vd.vd_append(self.cache, k, v, self.B)
+        idx = t.arange(units, device=self.device) * max(1, self.U // units)
+        kk = self.cache.k.view(self.U, self.cap, self.d)[idx]
+        vv = self.cache.v.view(self.U, self.cap, self.d)[idx]
+        vd.vd_evict_block(self.cache, self.N, None, self.B, self.variant, self.mu,
+                          self.rs if self.mu else None, None, None)
+        return kk, vv, self.N + self.B, self.N
+
+
+class Decode:
+    """Decode step at steady state: append one token, evict N + 1 -> N."""
+
+    def __init__(self, name, cfg, device, seed, mu, variant, n_tokens=8):
+        import torch
+        import paper_2609_23314_gb300 as vd
+        from paper_2609_23314_gb300 import workloads as wl
+        self.vd, self.torch = vd, torch
+        self.name, self.cfg, self.device = name, cfg, device
+        self.N, self.d = cfg["N"], cfg["head_dim"]
+        self.B = 1
+        self.cap = self.N + 1
+        self.cache = vd.Cache.empty(cfg["n_seq"], cfg["n_layer"], cfg["n_kv_head"], self.cap,
+                                    self.d, device=device)
+        self.U = self.cache.units
+        st = wl.stream_for(cfg, device=str(device), seed=seed)
+        kv = self.cache.k.view(self.U, self.cap, self.d), self.cache.v.view(self.U, self.cap, self.d)
+        wl.fill_rows(st, kv[0], kv[1], self.N, chunk_units=256, initial=True)
+        self.cache.len.fill_(self.N)
+        us = self.cache.unit_shape()
+        self.tokens = []
+        for _ in range(n_tokens):
+            k, v = st.next(1)
+            self.tokens.append((k.view(us + (1, self.d)).contiguous(),
+                                v.view(us + (1, self.d)).contiguous()))
+        self.mu, self.variant = mu, variant
+        self.rs = torch.zeros(us + (self.d,), dtype=torch.float64, device=device)
+        if mu == vd.VD_MU_RUNNING:
+            vd.vd_running_sum_init(self.cache, self.rs)
+        self.i = 0
+        self.launches_per_step = 4
+
+    def head_tokens_per_step(self):
+        return self.U * (self.N + 1)
+
+    def new_kept_buffers(self, k):
+        t = self.torch
+        return [t.empty(self.cache.unit_shape(), dtype=t.int32, device=self.device)
+                for _ in range(k)]
+
+    def step(self, kept=None, ev=None):
+        vd = self.vd
+        k, v = self.tokens[self.i % len(self.tokens)]
+        self.i += 1
+        vd.vd_append(self.cache, k, v, 1)
+        if ev is not None:
+            ev[0].record()
+        vd.vd_evict_decode(self.cache, self.N, None, self.variant, self.mu,
+                           self.rs if self.mu else None, kept, None, None)
+        if ev is not None:
+            ev[1].record()
+
+    def moved_rows(self, evicted_list):
+        total = 0
+        for e in evicted_list:
+            total += int((self.N - e.long()).sum().item())
+        return total / max(1, len(evicted_list))
+
+    def bytes_per_launch(self, moved_rows_total):
+        n, d = self.N + 1, self.d
+        v_read = self.U * n * d * 2
+        move = moved_rows_total * d * 2 * 2 * 2
+        extra = self.U * d * 8 * 2 if self.mu else 0
+        return v_read + move + extra, v_read + self.U * self.N * d * 2 * 2 * 2 + extra
+
+    def e2e_setup(self):
+        t = self.torch
+        us = self.cache.unit_shape()
+        self.h_tokens = [(k.cpu().pin_memory(), v.cpu().pin_memory()) for k, v in self.tokens[:2]]
+        self.d_k = t.empty(us + (1, self.d), dtype=t.bfloat16, device=self.device)
+        self.d_v = t.empty_like(self.d_k)
+        self.d_ev = t.empty(us, dtype=t.int32, device=self.device)
+        self.h_ev = t.empty(us, dtype=t.int32).pin_memory()
+        return 2 * self.d_k.numel() * 2, self.d_ev.numel() * 4
+
+    def e2e_step(self):
+        vd = self.vd
+        hk, hv = self.h_tokens[self.i % 2]
+        self.i += 1
+        self.d_k.copy_(hk, non_blocking=True)
+        self.d_v.copy_(hv, non_blocking=True)
+        vd.vd_append(self.cache, self.d_k, self.d_v, 1)
+        vd.vd_evict_decode(self.cache, self.N, None, self.variant, self.mu,
+                           self.rs if self.mu else None, self.d_ev, None, None)
+        self.h_ev.copy_(self.d_ev, non_blocking=True)
+
+    def oracle_sample(self, units):
+        t = self.torch
+        vd = self.vd
+        k, v = self.tokens[0]
+        vd.vd_append(self.cache, k, v, 1)
+        idx = t.arange(units, device=self.device) * max(1, self.U // units)
+        kk = self.cache.k.view(self.U, self.cap, self.d)[idx]
+        vv = self.cache.v.view(self.U, self.cap, self.d)[idx]
+        vd.vd_evict_decode(self.cache, self.N, None, self.variant, self.mu,
+                           self.rs if self.mu else None, None, None, None)
+        return kk, vv, self.N + 1, self.N
+
+
+def make_workload(name, device, seed, mu, variant):
+    from paper_2609_23314_gb300 import workloads as wl
+    _, cfg = wl.config(name)
+    if cfg["kind"] == "prefill":
+        return Prefill(name, cfg, device, seed, mu, variant)
+    if cfg["kind"] == "decode":
+        return Decode(name, cfg, device, seed, mu, variant)
+    # ratio budget: its largest event is a decode step at N = 25% of the final length
+    cfg = dict(cfg)
+    total = cfg["prompt"] + cfg["gen_tokens"]
+    cfg["N"] = wl.budget_at(cfg, total)
+    return Decode(name, cfg, device, seed, mu, variant)
+
+
+# ---------------------------------------------------------------------------
+# measurement
+# ---------------------------------------------------------------------------
+def measure_gpu(w, steps, warmup, device, e2e_steps):
+    import torch
+    for _ in range(warmup):
+        w.step()
+    torch.cuda.synchronize()
+    kept = w.new_kept_buffers(steps)
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+           for _ in range(steps)]
+    start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    barrier(device)
+    torch.cuda.synchronize()
+    clocks = ClockSampler(device.index if device.index is not None else 0)
+    clocks.start()
+    time.sleep(0.5)
+    t_begin = time.time()
+    start.record()
+    for i in range(steps):
+        w.step(kept[i], evs[i])
+    stop.record()
+    torch.cuda.synchronize()
+    clocks.mark(t_begin, time.time())
+    clk = clocks.stop()
+    barrier(device)
+    step_ms = start.elapsed_time(stop)
+    kern_ms = sum(a.elapsed_time(b) for a, b in evs) / steps
+    moved = w.moved_rows(kept)
+    # end to end through the C ABI with host buffers
+    bi, bo = w.e2e_setup()
+    for _ in range(min(3, warmup)):
+        w.e2e_step()
+    torch.cuda.synchronize()
+    barrier(device)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(e2e_steps):
+        w.e2e_step()
+    e1.record()
+    torch.cuda.synchronize()
+    e2e_ms = e0.elapsed_time(e1)
+    status = w.vd.vd_get_device_status()
+    if status != 0:
+        raise RuntimeError(f"device status {status}: {w.vd.vd_status_string(status)}")
+    return dict(step_ms=step_ms, kern_ms=kern_ms, moved=moved, clocks=clk, e2e_ms=e2e_ms,
+                bi=bi, bo=bo)
+
+
+def cpu_baseline(w, budget_s=2.0, max_units=64):
+    """The fp64 oracle (as it stands) on a bounded sample of the same events,
+    on every host core; returns the extrapolated head-tokens/s."""
+    import numpy as np
+    import oracle
+    orc = oracle.load()
+    cores = os.cpu_count() or 1
+    units = min(max_units, w.U)
+    kk, vv, n, N = w.oracle_sample(units)
+    k0 = kk.contiguous().view(w.torch.int16).cpu().numpy().view(np.uint16).copy()
+    v0 = vv.contiguous().view(w.torch.int16).cpu().numpy().view(np.uint16).copy()
+    lens = np.full(units, n, np.int32)
+    Ns = np.full(units, N, np.int32)
+    var = int(w.variant)
+    elapsed, events = 0.0, 0
+    while elapsed < budget_s or events == 0:
+        k, v = k0.copy(), v0.copy()
+        t0 = time.perf_counter()
+        orc.evict_units(k, v, lens, Ns, 1, var, nthreads=cores)
+        elapsed += time.perf_counter() - t0
+        events += 1
+    rate = units * n * events / elapsed
+    return {"value": rate, "unit": UNIT, "cores": cores, "kind": "oracle",
+            "sample": f"{units} of {w.U} units x {events} events of {w.name} at n={n} -> N={N}; "
+                      f"fp64 C oracle, one POSIX thread per core, {elapsed:.2f} s wall"}
+
+
+def run_vd(args):
+    import torch
+    import paper_2609_23314_gb300 as vd
+    from paper_2609_23314_gb300 import build as vd_build
+    ws, rank, local = dist_env()
+    if ws > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl")
+    else:
+        torch.cuda.set_device(0)
+    device = torch.device("cuda", torch.cuda.current_device())
+    if rank == 0:
+        vd_build.build()
+    barrier(device)
+    vd.load_library()
+    mu = vd.VD_MU_RUNNING if args.mu == "running" else vd.VD_MU_RECOMPUTE
+    variant = vd.VARIANTS[args.variant]
+    peak, peak_src = hbm_peak()
+    from paper_2609_23314_gb300 import workloads as wl
+
+    def one(name, steps):
+        _, cfg = wl.config(name)
+        w = make_workload(name, device, rank_seed(wl.BASE_SEED + cfg["index"], rank), mu, variant)
+        m = measure_gpu(w, steps, args.warmup, device, min(steps, args.e2e_steps))
+        step_ms = max_over_ranks(m["step_ms"], device) / steps
+        kern_ms = max_over_ranks(m["kern_ms"], device)
+        e2e_ms = max_over_ranks(m["e2e_ms"], device) / min(steps, args.e2e_steps)
+        tok = w.head_tokens_per_step()
+        alg, nominal = w.bytes_per_launch(m["moved"])
+        achieved = alg / (kern_ms / 1e3) / 1e9
+        res = {
+            "workload": name, "w": w, "m": m, "step_ms": step_ms, "kern_ms": kern_ms,
+            "value": tok * ws / (step_ms / 1e3),
+            "e2e": {"value": tok * ws / (e2e_ms / 1e3), "unit": UNIT,
+                    "h2d_bytes_per_step": m["bi"], "d2h_bytes_per_step": m["bo"]},
+            "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                         "frac": achieved / peak, "traffic": ncu_traffic(name),
+                         "kernel": f"vd::evict_kernel<{variant}, {'true' if isinstance(w, Decode) else 'false'}>",
+                         "algorithmic_bytes_per_launch": alg,
+                         "nominal_bytes_per_launch": nominal,
+                         "moved_rows_per_launch": m["moved"],
+                         "kernel_ms": kern_ms, "peak_source": peak_src + ", of measured"
+                         if "measured" in peak_src else peak_src},
+            "config": {"workload": name, **{k: cfg[k] for k in cfg if k not in ("index", "kind")},
+                       "mu": args.mu, "variant": args.variant,
+                       "l2": f"inputs larger than L2: cache {w.cache.k.numel() * 4 / 2**30:.2f} GiB "
+                             "of K+V, touched every step", "storage": "bf16"},
+        }
+        return res
+
+    primary = one(args.workload, args.steps)
+    base = None
+    if rank == 0 and not args.no_cpu_baseline:
+        base = cpu_baseline(primary["w"])
+    secondary = None
+    if args.secondary and args.secondary != args.workload:
+        secondary = one(args.secondary, max(3, args.steps // 20))
+    if rank == 0:
+        w = primary["w"]
+        line = {
+            "metric": METRIC, "value": primary["value"], "unit": UNIT, "n_gpus": ws,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": primary["step_ms"],
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": "f32", "data": "synthetic (seeded generators shaped like the paper's workloads)",
+            "config": primary["config"],
+            "roofline": primary["roofline"],
+            "e2e": primary["e2e"],
+            "clocks": primary["m"]["clocks"],
+            "gpu_launches": w.launches_per_step * args.steps,
+        }
+        if base is not None:
+            line["cpu_baseline"] = base
+        if secondary is not None:
+            line["secondary"] = {k: secondary[k] for k in ("workload", "value", "step_ms", "roofline",
+                                                           "e2e", "config")}
+            line["secondary"]["clocks"] = secondary["m"]["clocks"]
+        print(json.dumps(line), flush=True)
+    if ws > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+def run_reference(args):
+    """The CPU oracle as the reference arm: each step = one oracle pass over a
+    bounded sample of the workload's units at steady state."""
+    ws, rank, _ = dist_env()
+    if rank != 0:
+        return
+    import numpy as np
+    import torch
+    import oracle
+    from paper_2609_23314_gb300 import workloads as wl
+    orc = oracle.load()
+    name, cfg = wl.config(args.workload)
+    cores = os.cpu_count() or 1
+    d = cfg["head_dim"]
+    if cfg["kind"] == "prefill":
+        N, n = cfg["N"], cfg["N"] + cfg["B"]
+    else:
+        if cfg["kind"] == "ratio":
+            cfg["N"] = wl.budget_at(cfg, cfg["prompt"] + cfg["gen_tokens"])
+        N, n = cfg["N"], cfg["N"] + 1
+    units = max(1, min(wl.units_of(cfg), cores * 2))
+    st = wl.stream_for(cfg, device="cpu", units=units)
+    k, v = st.next(n, initial=True)
+    k0 = k.view(torch.int16).numpy().view(np.uint16).copy()
+    v0 = v.view(torch.int16).numpy().view(np.uint16).copy()
+    lens = np.full(units, n, np.int32)
+    Ns = np.full(units, N, np.int32)
+    var = {"l2": 0, "dir": 1, "norm": 2}[args.variant]
+    for _ in range(args.warmup):
+        kk, vv = k0.copy(), v0.copy()
+        orc.evict_units(kk, vv, lens, Ns, 1, var, nthreads=cores)
+    total = 0.0
+    for _ in range(args.steps):
+        kk, vv = k0.copy(), v0.copy()
+        t0 = time.perf_counter()
+        orc.evict_units(kk, vv, lens, Ns, 1, var, nthreads=cores)
+        total += time.perf_counter() - t0
+    ms = total / args.steps * 1e3
+    value = units * n / (ms / 1e3)
+    line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "impl": "reference",
+            "config": {"workload": name, "sample_units": units, "n": n, "N": N, "head_dim": d},
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
+                             "sample": f"{units} units of {name} per step at n={n} -> N={N}"},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def main(argv=None):
+    ap = argparse.ArgumentParser(description=__doc__.splitlines()[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=None)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["vd", "reference"], default="vd")
+    ap.add_argument("--workload", default="prefill_wide")
+    ap.add_argument("--secondary", default="decode_batched",
+                    help="a second workload measured into the same line ('' to skip)")
+    ap.add_argument("--mu", choices=["running", "recompute"], default="running")
+    ap.add_argument("--variant", choices=["l2", "dir", "norm"], default="l2")
+    ap.add_argument("--e2e-steps", type=int, default=50)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args(argv)
+    if args.warmup < 3:
+        ap.error("--warmup must be at least 3")
+    if args.steps is None:
+        args.steps = 5 if args.impl == "reference" else 1000
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_vd(args)
+
+
+if __name__ == "__main__":
+    main()

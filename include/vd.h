@@ -1,0 +1,167 @@
+/*
+ * vd.h -- C ABI of the GB300 (sm_103a) ValueDiff KV-cache eviction library
+ * (libvd.so).
+ *
+ * ValueDiff (Sec. 3.2, Eq. vd) scores every cached token of one
+ * (sequence, layer, KV head) "unit" by how far its value vector lies from the
+ * cache mean,  s_j = || v_j - mean ||_2,  mean = (1/n) sum_i v_i,  and the
+ * eviction policy pi_N of Sec. 2.1, Eq. (eviction) keeps the N highest-scoring
+ * tokens and gathers K and V to them.  pi_N runs at every block boundary of
+ * block prompt processing (Sec. 2.2, Eq. block_processing: cache N+B -> N)
+ * and at every decode step (abstract; Sec. 4 protocol: cache N+1 -> N).
+ *
+ * Conventions shared by every entry point
+ * ---------------------------------------
+ * - All buffers are caller-owned DEVICE memory unless stated otherwise.  The
+ *   library allocates no device memory; its only device state is one status
+ *   word per device (a static __device__ variable).
+ * - Calls are asynchronous on `stream` (a cudaStream_t; NULL = legacy default
+ *   stream).  Host-side validation happens before any launch: a call that
+ *   returns an error launched nothing and changed nothing.
+ * - Layout: K and V are bf16, [n_seq][n_layer][n_kv_head][capacity][head_dim]
+ *   row-major, so one unit's rows are contiguous.  Unit index
+ *   u = (seq * n_layer + layer) * n_kv_head + head.
+ * - len is a device int32 [n_seq]: every layer and head of a sequence holds
+ *   the same number of tokens.  Slots >= len are never read.
+ * - Top-N ties are broken toward the LOWER slot index (the earlier token; the
+ *   paper does not fix a tie rule).  Compaction keeps the surviving tokens in
+ *   their original (ascending slot) order.  Slots >= N after an eviction hold
+ *   unspecified bytes.
+ * - Anomalies found on the device (len > capacity, a per-sequence budget out
+ *   of range, a non-finite score, a decode call with more than one token over
+ *   budget) never trap: the kernel records the first one in the device status
+ *   word (read it with vd_get_device_status) and leaves the affected unit
+ *   untouched, except VD_ERR_NONFINITE, which is recorded while the unit is
+ *   still evicted with NaN scores ranked lowest.
+ * - Precision: scores are computed in fp32 from bf16 inputs; the cache mean
+ *   is accumulated with compensated fp32 sums (or kept as an fp64 running
+ *   sum) so that it is correct to about 1e-7 relative.
+ */
+#ifndef VD_H
+#define VD_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Same type as cudaStream_t. */
+typedef struct CUstream_st* vd_stream_t;
+
+typedef enum {
+  VD_OK = 0,
+  VD_ERR_INVALID_ARG = 1, /* null pointer, non-positive size, N out of range, ... */
+  VD_ERR_ALIGNMENT = 2,   /* K/V not 16-byte aligned, or head_dim % 8 != 0 */
+  VD_ERR_UNSUPPORTED = 3, /* shape beyond what the kernels handle (head_dim > 256,
+                             capacity too large for on-chip selection) */
+  VD_ERR_NONFINITE = 4,   /* device: a score was NaN or infinite */
+  VD_ERR_TIMEOUT = 5,     /* reserved: no kernel in this library waits on a flag */
+  VD_ERR_CUDA = 6,        /* a CUDA runtime call failed (launch error, ...) */
+  VD_ERR_DEVICE_LEN = 7,  /* device: len[s] out of [0, capacity], or len + B > capacity
+                             on append, or B > len in running-sum mode */
+  VD_ERR_DEVICE_BUDGET = 8, /* device: N_dev[s] out of [1, N], or a decode call found
+                               len > N + 1 */
+  VD_ERR_NO_DEVICE = 9    /* no CUDA device, or not an sm_103 device */
+} vd_status;
+
+/* Scoring rules of Sec. 3.2.  Higher scores are kept.
+ *   VD_SCORE_L2   s_j = || v_j - mean ||_2           (ValueDiff, Eq. vd)
+ *   VD_SCORE_DIR  s_j = 1 - cos(v_j, mean)           (ValueDiff-Dir; cos := 0 when
+ *                                                     v_j or the mean is zero)
+ *   VD_SCORE_NORM s_j = || v_j ||_2                  (ValueDiff-Norm; keeps the
+ *                                                     largest norms) */
+typedef enum { VD_SCORE_L2 = 0, VD_SCORE_DIR = 1, VD_SCORE_NORM = 2 } vd_variant;
+
+/* How the cache mean is obtained.
+ *   VD_MU_RECOMPUTE  sum every cached row at every event (reads V twice per
+ *                    event unless the cache slice fits on chip).
+ *   VD_MU_RUNNING    keep S = sum of the cached V rows as fp64 [unit][head_dim]
+ *                    across events; the mean is S / n.  V is read once.
+ *                    Not in the paper: an exact incremental form of its mean. */
+typedef enum { VD_MU_RECOMPUTE = 0, VD_MU_RUNNING = 1 } vd_mu_mode;
+
+typedef struct {
+  void* k;          /* bf16 device, [n_seq][n_layer][n_kv_head][capacity][head_dim], 16-B aligned */
+  void* v;          /* bf16 device, same layout as k, 16-B aligned */
+  int32_t* len;     /* device int32 [n_seq]: current number of cached tokens */
+  int32_t n_seq, n_layer, n_kv_head;
+  int32_t head_dim; /* multiple of 8, at most 256 */
+  int32_t capacity; /* slots per unit; the kernels size on-chip buffers by it */
+} vd_cache;
+
+/* Scores only (Eq. vd and its Sec. 3.2 variants), mean recomputed from the
+ * cache.  scores_out: fp32 device [n_seq][n_layer][n_kv_head][capacity]; rows
+ * j < len[s] are written, rows >= len[s] untouched.  The cache is not
+ * modified. */
+vd_status vd_score(const vd_cache* c, vd_variant var, float* scores_out, vd_stream_t stream);
+
+/* Block-boundary eviction (Sec. 2.2, Eq. block_processing): the caller has
+ * already appended B rows (len = old + B).  For every unit whose sequence has
+ * len > N_s: score, keep the top N_s (Sec. 2.1, Eq. eviction), compact K and V
+ * in place in ascending slot order and set len = N_s.  Sequences with
+ * len <= N_s are left as they are ("evict whenever the cache exceeds N").
+ *   N            scalar budget, 1 <= N <= capacity; also the row stride of
+ *                kept_idx_out and the upper bound of N_dev values.
+ *   N_dev        nullable device int32 [n_seq]: per-sequence budgets N_s in
+ *                [1, N] (e.g. a budget that grows with length); NULL -> N_s = N.
+ *   B            rows appended since the previous call, 0 <= B <= capacity;
+ *                used only by VD_MU_RUNNING.
+ *   running_sum  fp64 device [n_seq][n_layer][n_kv_head][head_dim], required
+ *                when mu == VD_MU_RUNNING: on entry the sum of V rows
+ *                [0, len - B) (the rows present after the previous call), on
+ *                exit the sum of the rows [0, new len).  Initialise it with
+ *                vd_running_sum_init.  Ignored for VD_MU_RECOMPUTE.
+ *   kept_idx_out nullable int32 device [n_seq][n_layer][n_kv_head][N]: the
+ *                pre-eviction slot of every surviving token, ascending; for a
+ *                unit that did not evict, 0..len-1 followed by -1.
+ *   scores_out   nullable fp32 device [..][capacity]: the scores of the
+ *                pre-eviction rows, written only for units that evicted. */
+vd_status vd_evict_block(const vd_cache* c, int32_t N, const int32_t* N_dev, int32_t B,
+                         vd_variant var, vd_mu_mode mu, double* running_sum,
+                         int32_t* kept_idx_out, float* scores_out, vd_stream_t stream);
+
+/* Decode-step eviction (per-token eviction of the abstract and the Sec. 4
+ * protocol; Eq. block_processing with B = 1): the caller has appended one
+ * token, so len <= N_s + 1.  Units with len = N_s + 1 evict exactly one token
+ * (the lowest score; among tied minima the highest slot) and compact.
+ * Arguments as in vd_evict_block with B = 1, plus
+ *   evicted_out  nullable int32 device [n_seq][n_layer][n_kv_head]: the
+ *                evicted pre-eviction slot, or -1 where nothing was evicted.
+ * A sequence found with len > N_s + 1 is left untouched and records
+ * VD_ERR_DEVICE_BUDGET. */
+vd_status vd_evict_decode(const vd_cache* c, int32_t N, const int32_t* N_dev, vd_variant var,
+                          vd_mu_mode mu, double* running_sum, int32_t* evicted_out,
+                          int32_t* kept_idx_out, float* scores_out, vd_stream_t stream);
+
+/* Append B new rows per unit at slots [len, len + B) and set len += B (the
+ * block append of Eq. block_processing).  k_new, v_new: bf16 device
+ * [n_seq][n_layer][n_kv_head][B][head_dim], 16-B aligned.  A sequence with
+ * len + B > capacity is left untouched and records VD_ERR_DEVICE_LEN.  The
+ * running sum, if any, is NOT touched here: vd_evict_* adds the appended rows
+ * (pass the same B). */
+vd_status vd_append(const vd_cache* c, const void* k_new, const void* v_new, int32_t B,
+                    vd_stream_t stream);
+
+/* running_sum[u][:] = sum of V rows [0, len) of unit u, from scratch (fp64
+ * [n_seq][n_layer][n_kv_head][head_dim], device). */
+vd_status vd_running_sum_init(const vd_cache* c, double* running_sum, vd_stream_t stream);
+
+/* Device scratch the calls need beyond their arguments: always 0 (the fused
+ * kernels keep every intermediate on chip). */
+size_t vd_workspace_size(const vd_cache* c);
+
+/* Static English text for a status code (never NULL). */
+const char* vd_status_string(vd_status st);
+
+/* Synchronises `stream`, returns the first device-side anomaly recorded since
+ * the previous call (VD_OK if none) and clears it.  A sticky CUDA error on
+ * the stream is returned as VD_ERR_CUDA. */
+vd_status vd_get_device_status(vd_stream_t stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* VD_H */

@@ -1,0 +1,414 @@
+// vd_api.cu -- host side of libvd.so: the C ABI declared in include/vd.h.
+//
+// Validates arguments before any launch, sizes the thread-block cluster per
+// unit, launches the fused eviction kernel with cudaLaunchKernelExC on the
+// caller's stream, and owns the device status word (a static __device__
+// variable: the library allocates no device memory).
+#include <cuda_runtime.h>
+
+#include <climits>
+#include <cstdint>
+#include <cstdlib>
+#include <mutex>
+
+#include "vd.h"
+#include "vd_evict.cuh"
+
+namespace vd {
+const void* evict_kernel_l2(bool decode);
+const void* evict_kernel_dir(bool decode);
+const void* evict_kernel_norm(bool decode);
+}  // namespace vd
+
+using vd::kThreads;
+
+// First device-side anomaly since the last vd_get_device_status (0 = none).
+static __device__ unsigned g_vd_status;
+
+// ---------------------------------------------------------------------------
+// small kernels: append (Eq. block_processing's concatenation), length
+// update after an eviction, and the from-scratch running sum
+// ---------------------------------------------------------------------------
+__global__ void vd_append_kernel(uint16_t* __restrict__ k, uint16_t* __restrict__ v,
+                                 const uint16_t* __restrict__ kn, const uint16_t* __restrict__ vn,
+                                 const int32_t* __restrict__ len, int units_per_seq,
+                                 long long n_units, int cap, int d, int B, unsigned* status) {
+  const int d8 = d >> 3;
+  const long long total = n_units * (long long)B * d8;
+  for (long long idx = blockIdx.x * (long long)blockDim.x + threadIdx.x; idx < total;
+       idx += (long long)gridDim.x * blockDim.x) {
+    const int c = (int)(idx % d8);
+    const long long ub = idx / d8;
+    const int b = (int)(ub % B);
+    const long long u = ub / B;
+    const int n = len[u / units_per_seq];
+    if (n < 0 || n > cap - B) {
+      if (b == 0 && c == 0 && u % units_per_seq == 0) vd::record_status(status, vd::kStDeviceLen);
+      continue;
+    }
+    const size_t src = (size_t)ub * d + (size_t)c * 8;
+    const size_t dst = ((size_t)u * cap + (size_t)(n + b)) * d + (size_t)c * 8;
+    vd::st16(k + dst, vd::ld_cg16(kn + src));
+    vd::st16(v + dst, vd::ld_cg16(vn + src));
+  }
+}
+
+__global__ void vd_len_add_kernel(int32_t* len, int n_seq, int cap, int B) {
+  const int s = blockIdx.x * blockDim.x + threadIdx.x;
+  if (s >= n_seq) return;
+  const int n = len[s];
+  if (n >= 0 && n <= cap - B) len[s] = n + B;
+}
+
+// Mirrors the eviction kernel's per-sequence decision exactly.
+__global__ void vd_len_clamp_kernel(int32_t* len, const int32_t* N_dev, int N, int n_seq,
+                                    int cap, int B, int running, int decode) {
+  const int s = blockIdx.x * blockDim.x + threadIdx.x;
+  if (s >= n_seq) return;
+  const int n = len[s];
+  const int Nb = N_dev ? N_dev[s] : N;
+  if (n < 0 || n > cap || (running && B > n)) return;
+  if (Nb < 1 || Nb > N || n <= Nb) return;
+  if (decode && n > Nb + 1) return;
+  len[s] = Nb;
+}
+
+__global__ void __launch_bounds__(kThreads) vd_rsum_init_kernel(const uint16_t* __restrict__ v,
+                                                                const int32_t* __restrict__ len,
+                                                                double* rs, int units_per_seq,
+                                                                int cap, int d, int lpr,
+                                                                unsigned* status) {
+  __shared__ float hi[256], lo[256];
+  const int u = blockIdx.x;
+  const int n = len[u / units_per_seq];
+  if (n < 0 || n > cap) {
+    if (threadIdx.x == 0 && u % units_per_seq == 0) vd::record_status(status, vd::kStDeviceLen);
+    return;
+  }
+  hi[threadIdx.x] = 0.f;
+  lo[threadIdx.x] = 0.f;
+  __syncthreads();
+  const uint16_t* vb = v + (size_t)u * cap * d;
+  vd::accumulate_rows(vb, d, 0, d >> 3, lpr, n,
+                      [&](int i, int& row, float& sign) { row = i; sign = 1.f; }, hi, lo);
+  if ((int)threadIdx.x < d)
+    rs[(size_t)u * d + threadIdx.x] = (double)hi[threadIdx.x] + (double)lo[threadIdx.x];
+}
+
+// ---------------------------------------------------------------------------
+// per-device state
+// ---------------------------------------------------------------------------
+namespace {
+
+struct DeviceState {
+  bool ready = false;
+  unsigned* status = nullptr;
+  int sms = 0;
+  int smem_optin = 0;
+};
+
+constexpr int kMaxDevices = 64;
+std::mutex g_mu;
+DeviceState g_dev[kMaxDevices];
+
+const void* evict_kernel(vd_variant var, bool decode) {
+  switch (var) {
+    case VD_SCORE_L2: return vd::evict_kernel_l2(decode);
+    case VD_SCORE_DIR: return vd::evict_kernel_dir(decode);
+    default: return vd::evict_kernel_norm(decode);
+  }
+}
+
+vd_status device_state(DeviceState** out) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) {
+    cudaGetLastError();
+    return VD_ERR_NO_DEVICE;
+  }
+  std::lock_guard<std::mutex> lk(g_mu);
+  DeviceState& st = g_dev[dev];
+  if (!st.ready) {
+    cudaDeviceProp p;
+    if (cudaGetDeviceProperties(&p, dev) != cudaSuccess) {
+      cudaGetLastError();
+      return VD_ERR_NO_DEVICE;
+    }
+    if (p.major != 10 || p.minor != 3) return VD_ERR_NO_DEVICE;  // built for sm_103a only
+    void* ptr = nullptr;
+    if (cudaGetSymbolAddress(&ptr, g_vd_status) != cudaSuccess) return VD_ERR_CUDA;
+    st.status = static_cast<unsigned*>(ptr);
+    st.sms = p.multiProcessorCount;
+    st.smem_optin = (int)p.sharedMemPerBlockOptin;
+    for (int var = 0; var < 3; ++var)
+      for (int dec = 0; dec < 2; ++dec) {
+        const void* kern = evict_kernel((vd_variant)var, dec != 0);
+        if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 st.smem_optin) != cudaSuccess ||
+            cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) !=
+                cudaSuccess)
+          return VD_ERR_CUDA;
+      }
+    st.ready = true;
+  }
+  *out = &st;
+  return VD_OK;
+}
+
+vd_status validate_cache(const vd_cache* c) {
+  if (!c || !c->k || !c->v || !c->len) return VD_ERR_INVALID_ARG;
+  if (c->n_seq < 1 || c->n_layer < 1 || c->n_kv_head < 1 || c->capacity < 1 || c->head_dim < 1)
+    return VD_ERR_INVALID_ARG;
+  if (c->head_dim % 8 != 0) return VD_ERR_ALIGNMENT;
+  if (c->head_dim > 256) return VD_ERR_UNSUPPORTED;
+  if ((reinterpret_cast<uintptr_t>(c->k) | reinterpret_cast<uintptr_t>(c->v)) & 15u)
+    return VD_ERR_ALIGNMENT;
+  const long long units = (long long)c->n_seq * c->n_layer * c->n_kv_head;
+  if (units * 16 > INT_MAX) return VD_ERR_UNSUPPORTED;  // grid of units x cluster CTAs
+  return VD_OK;
+}
+
+int lanes_per_row(int d) {
+  int p = 1;
+  while (p < d / 8) p <<= 1;
+  return p;
+}
+
+bool cluster_fits(const void* kern, long long units, int c, size_t smem) {
+  if (c == 1) return true;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)(units * c));
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = smem;
+  cudaLaunchAttribute attr;
+  attr.id = cudaLaunchAttributeClusterDimension;
+  attr.val.clusterDim.x = (unsigned)c;
+  attr.val.clusterDim.y = 1;
+  attr.val.clusterDim.z = 1;
+  cfg.attrs = &attr;
+  cfg.numAttrs = 1;
+  int ncl = 0;
+  if (cudaOccupancyMaxActiveClusters(&ncl, kern, &cfg) != cudaSuccess) {
+    cudaGetLastError();
+    return false;
+  }
+  return ncl > 0;
+}
+
+// CTAs per unit: enough CTAs to cover the GPU several times over, while each
+// CTA still moves row segments of at least 64 bytes of [K | V].  The
+// environment variable VD_CLUSTER_SIZE (1, 2, 4, 8 or 16) overrides the
+// choice, for tuning.
+int choose_cluster(const void* kern, long long units, int d, size_t smem, const DeviceState& st) {
+  const int total_chunks = 2 * (d / 8);
+  int max_c = 1;
+  for (int c = 2; c <= 16; c *= 2)
+    if (total_chunks % c == 0 && total_chunks / c >= 4) max_c = c;
+  int c = 1;
+  const char* env = std::getenv("VD_CLUSTER_SIZE");
+  const int want = env ? std::atoi(env) : 0;
+  if (want >= 1 && want <= 16 && (want & (want - 1)) == 0 && total_chunks % want == 0) {
+    c = want;
+  } else {
+    int occ = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, kern, kThreads, smem) != cudaSuccess)
+      cudaGetLastError();
+    if (occ < 1) occ = 1;
+    const long long slots = (long long)st.sms * occ;
+    while (c < max_c && units * c < 4 * slots) c <<= 1;
+  }
+  while (c > 1 && !cluster_fits(kern, units, c, smem)) c >>= 1;
+  return c;
+}
+
+vd_status launch(const void* kern, long long units, int c, size_t smem, const vd::EvictArgs& a,
+                 cudaStream_t s) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)(units * c));
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr;
+  attr.id = cudaLaunchAttributeClusterDimension;
+  attr.val.clusterDim.x = (unsigned)c;
+  attr.val.clusterDim.y = 1;
+  attr.val.clusterDim.z = 1;
+  cfg.attrs = &attr;
+  cfg.numAttrs = 1;
+  void* args[] = {const_cast<vd::EvictArgs*>(&a)};
+  if (cudaLaunchKernelExC(&cfg, kern, args) != cudaSuccess) {
+    cudaGetLastError();
+    return VD_ERR_CUDA;
+  }
+  return VD_OK;
+}
+
+size_t evict_smem(int capacity, bool decode) {
+  size_t b = sizeof(vd::Smem);
+  if (!decode) b += (size_t)capacity * 8;
+  return (b + 15) & ~(size_t)15;
+}
+
+vd_status run(const vd_cache* c, int32_t N, const int32_t* N_dev, int32_t B, vd_variant var,
+              vd_mu_mode mu, double* running_sum, int32_t* evicted_out, int32_t* kept_idx_out,
+              float* scores_out, cudaStream_t s, bool decode, bool score_only) {
+  vd_status r = validate_cache(c);
+  if (r != VD_OK) return r;
+  if (var != VD_SCORE_L2 && var != VD_SCORE_DIR && var != VD_SCORE_NORM) return VD_ERR_INVALID_ARG;
+  if (mu != VD_MU_RECOMPUTE && mu != VD_MU_RUNNING) return VD_ERR_INVALID_ARG;
+  if (!score_only) {
+    if (N < 1 || N > c->capacity) return VD_ERR_INVALID_ARG;
+    if (B < 0 || B > c->capacity) return VD_ERR_INVALID_ARG;
+    if (mu == VD_MU_RUNNING && !running_sum) return VD_ERR_INVALID_ARG;
+  } else if (!scores_out) {
+    return VD_ERR_INVALID_ARG;
+  }
+  DeviceState* st = nullptr;
+  r = device_state(&st);
+  if (r != VD_OK) return r;
+
+  // score-only uses the decode instantiation: it needs no per-token buffers
+  const bool small = decode || score_only;
+  const size_t smem = evict_smem(c->capacity, small);
+  if (smem > (size_t)st->smem_optin) return VD_ERR_UNSUPPORTED;
+  const void* kern = evict_kernel(var, small);
+  const long long units = (long long)c->n_seq * c->n_layer * c->n_kv_head;
+
+  vd::EvictArgs a;
+  a.k = static_cast<uint16_t*>(c->k);
+  a.v = static_cast<uint16_t*>(c->v);
+  a.len = c->len;
+  a.N_dev = score_only ? nullptr : N_dev;
+  a.running_sum = running_sum;
+  a.kept_out = score_only ? nullptr : kept_idx_out;
+  a.evicted_out = decode ? evicted_out : nullptr;
+  a.scores_out = scores_out;
+  a.status = st->status;
+  a.units_per_seq = c->n_layer * c->n_kv_head;
+  a.d = c->head_dim;
+  a.lpr = lanes_per_row(c->head_dim);
+  a.capacity = c->capacity;
+  a.N = score_only ? 1 : N;
+  a.B = decode ? 1 : B;
+  a.mu_running = (!score_only && mu == VD_MU_RUNNING) ? 1 : 0;
+  a.score_only = score_only ? 1 : 0;
+  a.cluster = choose_cluster(kern, units, c->head_dim, smem, *st);
+
+  r = launch(kern, units, a.cluster, smem, a, s);
+  if (r != VD_OK || score_only) return r;
+  const int threads = 256;
+  vd_len_clamp_kernel<<<(c->n_seq + threads - 1) / threads, threads, 0, s>>>(
+      c->len, N_dev, N, c->n_seq, c->capacity, a.B, a.mu_running, decode ? 1 : 0);
+  if (cudaGetLastError() != cudaSuccess) return VD_ERR_CUDA;
+  return VD_OK;
+}
+
+}  // namespace
+
+// ---------------------------------------------------------------------------
+// C ABI
+// ---------------------------------------------------------------------------
+extern "C" {
+
+vd_status vd_score(const vd_cache* c, vd_variant var, float* scores_out, vd_stream_t stream) {
+  return run(c, 1, nullptr, 0, var, VD_MU_RECOMPUTE, nullptr, nullptr, nullptr, scores_out,
+             reinterpret_cast<cudaStream_t>(stream), false, true);
+}
+
+vd_status vd_evict_block(const vd_cache* c, int32_t N, const int32_t* N_dev, int32_t B,
+                         vd_variant var, vd_mu_mode mu, double* running_sum,
+                         int32_t* kept_idx_out, float* scores_out, vd_stream_t stream) {
+  return run(c, N, N_dev, B, var, mu, running_sum, nullptr, kept_idx_out, scores_out,
+             reinterpret_cast<cudaStream_t>(stream), false, false);
+}
+
+vd_status vd_evict_decode(const vd_cache* c, int32_t N, const int32_t* N_dev, vd_variant var,
+                          vd_mu_mode mu, double* running_sum, int32_t* evicted_out,
+                          int32_t* kept_idx_out, float* scores_out, vd_stream_t stream) {
+  return run(c, N, N_dev, 1, var, mu, running_sum, evicted_out, kept_idx_out, scores_out,
+             reinterpret_cast<cudaStream_t>(stream), true, false);
+}
+
+vd_status vd_append(const vd_cache* c, const void* k_new, const void* v_new, int32_t B,
+                    vd_stream_t stream) {
+  vd_status r = validate_cache(c);
+  if (r != VD_OK) return r;
+  if (!k_new || !v_new || B < 0 || B > c->capacity) return VD_ERR_INVALID_ARG;
+  if ((reinterpret_cast<uintptr_t>(k_new) | reinterpret_cast<uintptr_t>(v_new)) & 15u)
+    return VD_ERR_ALIGNMENT;
+  if (B == 0) return VD_OK;
+  DeviceState* st = nullptr;
+  r = device_state(&st);
+  if (r != VD_OK) return r;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  const long long units = (long long)c->n_seq * c->n_layer * c->n_kv_head;
+  const long long work = units * B * (c->head_dim / 8);
+  const long long want = (work + 255) / 256;
+  const int blocks = (int)(want < (long long)st->sms * 32 ? want : (long long)st->sms * 32);
+  vd_append_kernel<<<blocks, 256, 0, s>>>(
+      static_cast<uint16_t*>(c->k), static_cast<uint16_t*>(c->v),
+      static_cast<const uint16_t*>(k_new), static_cast<const uint16_t*>(v_new), c->len,
+      c->n_layer * c->n_kv_head, units, c->capacity, c->head_dim, B, st->status);
+  vd_len_add_kernel<<<(c->n_seq + 255) / 256, 256, 0, s>>>(c->len, c->n_seq, c->capacity, B);
+  if (cudaGetLastError() != cudaSuccess) return VD_ERR_CUDA;
+  return VD_OK;
+}
+
+vd_status vd_running_sum_init(const vd_cache* c, double* running_sum, vd_stream_t stream) {
+  vd_status r = validate_cache(c);
+  if (r != VD_OK) return r;
+  if (!running_sum) return VD_ERR_INVALID_ARG;
+  DeviceState* st = nullptr;
+  r = device_state(&st);
+  if (r != VD_OK) return r;
+  const long long units = (long long)c->n_seq * c->n_layer * c->n_kv_head;
+  vd_rsum_init_kernel<<<(unsigned)units, kThreads, 0, reinterpret_cast<cudaStream_t>(stream)>>>(
+      static_cast<const uint16_t*>(c->v), c->len, running_sum, c->n_layer * c->n_kv_head,
+      c->capacity, c->head_dim, lanes_per_row(c->head_dim), st->status);
+  if (cudaGetLastError() != cudaSuccess) return VD_ERR_CUDA;
+  return VD_OK;
+}
+
+size_t vd_workspace_size(const vd_cache* c) {
+  (void)c;
+  return 0;
+}
+
+const char* vd_status_string(vd_status st) {
+  switch (st) {
+    case VD_OK: return "ok";
+    case VD_ERR_INVALID_ARG: return "invalid argument";
+    case VD_ERR_ALIGNMENT: return "misaligned pointer or head_dim not a multiple of 8";
+    case VD_ERR_UNSUPPORTED: return "unsupported shape";
+    case VD_ERR_NONFINITE: return "non-finite score on the device";
+    case VD_ERR_TIMEOUT: return "device wait timed out";
+    case VD_ERR_CUDA: return "CUDA runtime error";
+    case VD_ERR_DEVICE_LEN: return "device: sequence length out of range";
+    case VD_ERR_DEVICE_BUDGET: return "device: budget out of range or decode over budget";
+    case VD_ERR_NO_DEVICE: return "no sm_103 CUDA device";
+    default: return "unknown status";
+  }
+}
+
+vd_status vd_get_device_status(vd_stream_t stream) {
+  DeviceState* st = nullptr;
+  vd_status r = device_state(&st);
+  if (r != VD_OK) return r;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if (cudaStreamSynchronize(s) != cudaSuccess) {
+    cudaGetLastError();
+    return VD_ERR_CUDA;
+  }
+  unsigned w = 0;
+  const unsigned z = 0;
+  if (cudaMemcpyFromSymbolAsync(&w, g_vd_status, sizeof w, 0, cudaMemcpyDeviceToHost, s) !=
+          cudaSuccess ||
+      cudaMemcpyToSymbolAsync(g_vd_status, &z, sizeof z, 0, cudaMemcpyHostToDevice, s) !=
+          cudaSuccess ||
+      cudaStreamSynchronize(s) != cudaSuccess) {
+    cudaGetLastError();
+    return VD_ERR_CUDA;
+  }
+  return static_cast<vd_status>(w);
+}
+
+}  // extern "C"

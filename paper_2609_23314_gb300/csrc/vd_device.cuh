@@ -1,0 +1,198 @@
+// vd_device.cuh -- device-side building blocks of the GB300 (sm_103a) ValueDiff
+// eviction kernels: bf16 unpacking, compensated fp32 sums, thread-block
+// cluster primitives (distributed shared memory, hardware cluster barrier) and
+// block-wide scans/reductions for a 256-thread CTA.
+#pragma once
+
+#include <cstdint>
+#include <cuda_runtime.h>
+
+namespace vd {
+
+constexpr int kThreads = 256;
+constexpr int kWarps = kThreads / 32;
+constexpr unsigned kFull = 0xffffffffu;
+
+// Device status codes (the values of vd_status in include/vd.h).
+constexpr unsigned kStNonfinite = 4;
+constexpr unsigned kStDeviceLen = 7;
+constexpr unsigned kStDeviceBudget = 8;
+
+// First anomaly wins; later ones are dropped.  Never traps.
+__device__ __forceinline__ void record_status(unsigned* st, unsigned code) {
+  atomicCAS(st, 0u, code);
+}
+
+// ---------------------------------------------------------------------------
+// bf16 <-> fp32.  A bf16 value is the upper half of an fp32 bit pattern, so
+// widening is a shift; eight values arrive per 16-byte vector.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ void unpack8(const uint4& q, float (&x)[8]) {
+  x[0] = __uint_as_float(q.x << 16);
+  x[1] = __uint_as_float(q.x & 0xffff0000u);
+  x[2] = __uint_as_float(q.y << 16);
+  x[3] = __uint_as_float(q.y & 0xffff0000u);
+  x[4] = __uint_as_float(q.z << 16);
+  x[5] = __uint_as_float(q.z & 0xffff0000u);
+  x[6] = __uint_as_float(q.w << 16);
+  x[7] = __uint_as_float(q.w & 0xffff0000u);
+}
+
+__device__ __forceinline__ uint4 ld_cg16(const void* p) {
+  uint4 r;
+  asm volatile("ld.global.cg.v4.u32 {%0,%1,%2,%3}, [%4];"
+               : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w)
+               : "l"(p));
+  return r;
+}
+
+__device__ __forceinline__ void st16(void* p, const uint4& v) {
+  asm volatile("st.global.v4.u32 [%0], {%1,%2,%3,%4};" ::"l"(p), "r"(v.x), "r"(v.y), "r"(v.z),
+               "r"(v.w)
+               : "memory");
+}
+
+// ---------------------------------------------------------------------------
+// Double-float (hi + lo) sums in fp32 arithmetic.  Each element enters with
+// Knuth's TwoSum, whose rounding error is exact and collected in lo, so a sum
+// over thousands of bf16 rows keeps ~2^-44 relative accuracy without fp64 in
+// the inner loop (fp64 throughput on GB300 is a small fraction of fp32).
+// ---------------------------------------------------------------------------
+struct ff {
+  float hi, lo;
+};
+
+__device__ __forceinline__ void ff_accumulate(float& hi, float& lo, float x) {
+  const float s = hi + x;
+  const float bb = s - hi;
+  lo += (hi - (s - bb)) + (x - bb);
+  hi = s;
+}
+
+__device__ __forceinline__ ff ff_add(ff a, ff b) {
+  const float s = a.hi + b.hi;
+  const float v = s - a.hi;
+  float e = (a.hi - (s - v)) + (b.hi - v);
+  e += a.lo + b.lo;
+  const float hi = s + e;
+  return {hi, e - (hi - s)};
+}
+
+__device__ __forceinline__ ff ff_shfl_xor(ff a, int off) {
+  return {__shfl_xor_sync(kFull, a.hi, off), __shfl_xor_sync(kFull, a.lo, off)};
+}
+
+// ---------------------------------------------------------------------------
+// Thread-block clusters: all CTAs of one (sequence, layer, head) unit form one
+// cluster.  Shared memory of a peer CTA is addressed through `mapa`; the
+// hardware cluster barrier (release/acquire) orders those accesses.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ unsigned cluster_ctarank() {
+  unsigned r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+
+__device__ __forceinline__ unsigned cluster_id_x() {
+  unsigned r;
+  asm volatile("mov.u32 %0, %%clusterid.x;" : "=r"(r));
+  return r;
+}
+
+__device__ __forceinline__ void cluster_arrive() {
+  asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ void cluster_wait() {
+  asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ void cluster_sync() {
+  cluster_arrive();
+  cluster_wait();
+}
+
+__device__ __forceinline__ uint32_t smem_addr(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+__device__ __forceinline__ uint32_t mapa(uint32_t addr, unsigned rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(addr), "r"(rank));
+  return r;
+}
+
+__device__ __forceinline__ void st_cluster_u32(uint32_t addr, uint32_t v) {
+  asm volatile("st.shared::cluster.u32 [%0], %1;" ::"r"(addr), "r"(v) : "memory");
+}
+
+__device__ __forceinline__ uint32_t ld_cluster_u32(uint32_t addr) {
+  uint32_t v;
+  asm volatile("ld.shared::cluster.u32 %0, [%1];" : "=r"(v) : "r"(addr) : "memory");
+  return v;
+}
+
+__device__ __forceinline__ uint64_t ld_cluster_u64(uint32_t addr) {
+  uint64_t v;
+  asm volatile("ld.shared::cluster.u64 %0, [%1];" : "=l"(v) : "r"(addr) : "memory");
+  return v;
+}
+
+__device__ __forceinline__ float ld_cluster_f32(uint32_t addr) {
+  return __uint_as_float(ld_cluster_u32(addr));
+}
+
+// ---------------------------------------------------------------------------
+// Block-wide helpers for a kThreads-thread CTA.  `sh` is kWarps ints of shared
+// scratch; every helper ends with a barrier so `sh` can be reused at once.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ int block_exclusive_scan(int v, int* sh, int& total) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  int x = v;
+#pragma unroll
+  for (int off = 1; off < 32; off <<= 1) {
+    const int y = __shfl_up_sync(kFull, x, off);
+    if (lane >= off) x += y;
+  }
+  if (lane == 31) sh[warp] = x;
+  __syncthreads();
+  if (warp == 0) {
+    int t = lane < kWarps ? sh[lane] : 0;
+#pragma unroll
+    for (int off = 1; off < kWarps; off <<= 1) {
+      const int y = __shfl_up_sync(kFull, t, off);
+      if (lane >= off) t += y;
+    }
+    if (lane < kWarps) sh[lane] = t;
+  }
+  __syncthreads();
+  const int res = (warp ? sh[warp - 1] : 0) + x - v;
+  total = sh[kWarps - 1];
+  __syncthreads();
+  return res;
+}
+
+__device__ __forceinline__ uint64_t warp_min_u64(uint64_t v) {
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+    const uint64_t o = __shfl_xor_sync(kFull, v, off);
+    v = o < v ? o : v;
+  }
+  return v;
+}
+
+// Deterministic (fixed-order) block sum of one float per thread.
+__device__ __forceinline__ float block_sum_f32(float v, float* sh) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) v += __shfl_xor_sync(kFull, v, off);
+  if (lane == 0) sh[warp] = v;
+  __syncthreads();
+  float t = 0.f;
+#pragma unroll
+  for (int w = 0; w < kWarps; ++w) t += sh[w];
+  __syncthreads();
+  return t;
+}
+
+}  // namespace vd

@@ -1,0 +1,10 @@
+// vd_evict_norm.cu -- instantiates the fused eviction kernel for one scoring
+// rule (compiled separately so the translation units build in parallel).
+#include "vd_evict.cuh"
+
+namespace vd {
+const void* evict_kernel_norm(bool decode) {
+  return decode ? reinterpret_cast<const void*>(&evict_kernel<2, true>)
+                : reinterpret_cast<const void*>(&evict_kernel<2, false>);
+}
+}  // namespace vd
