@@ -400,9 +400,11 @@ class Decode:
         return kk, vv, self.N + 1, self.N
 
 
-def make_workload(name, device, seed, mu, variant):
+def make_workload(name, device, seed, mu, variant, n_seq=None):
     from paper_2609_23314_gb300 import workloads as wl
     _, cfg = wl.config(name)
+    if n_seq:
+        cfg["n_seq"] = n_seq
     if cfg["kind"] == "prefill":
         return Prefill(name, cfg, device, seed, mu, variant)
     if cfg["kind"] == "decode":
@@ -513,7 +515,10 @@ def run_vd(args):
 
     def one(name, steps):
         _, cfg = wl.config(name)
-        w = make_workload(name, device, rank_seed(wl.BASE_SEED + cfg["index"], rank), mu, variant)
+        if args.n_seq:
+            cfg["n_seq"] = args.n_seq
+        w = make_workload(name, device, rank_seed(wl.BASE_SEED + cfg["index"], rank), mu, variant,
+                          args.n_seq)
         m = measure_gpu(w, steps, args.warmup, device, min(steps, args.e2e_steps))
         step_ms = max_over_ranks(m["step_ms"], device) / steps
         kern_ms = max_over_ranks(m["kern_ms"], device)
@@ -546,7 +551,7 @@ def run_vd(args):
     if rank == 0 and not args.no_cpu_baseline:
         base = cpu_baseline(primary["w"])
     secondary = None
-    if args.secondary and args.secondary != args.workload:
+    if args.secondary not in ("", "none") and args.secondary != args.workload:
         secondary = one(args.secondary, max(3, args.steps // 20))
     if rank == 0:
         w = primary["w"]
@@ -635,6 +640,8 @@ def main(argv=None):
     ap.add_argument("--mu", choices=["running", "recompute"], default="running")
     ap.add_argument("--variant", choices=["l2", "dir", "norm"], default="l2")
     ap.add_argument("--e2e-steps", type=int, default=50)
+    ap.add_argument("--n-seq", type=int, default=None,
+                    help="override the workload's number of sequences (smaller profiling cases)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     args = ap.parse_args(argv)
     if args.warmup < 3:
