@@ -7,6 +7,7 @@
 #include <cuda_runtime.h>
 
 #include <climits>
+#include <cmath>
 #include <cstdint>
 #include <cstdlib>
 #include <mutex>
@@ -78,21 +79,20 @@ __global__ void __launch_bounds__(kThreads) vd_rsum_init_kernel(const uint16_t* 
                                                                 double* rs, int units_per_seq,
                                                                 int cap, int d, int lpr,
                                                                 unsigned* status) {
-  __shared__ float hi[256], lo[256];
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  vd::Smem& S = *reinterpret_cast<vd::Smem*>(smem_raw);
+  const uint32_t ring = vd::smem_addr(smem_raw + vd::smem_layout(cap, 1, false).ring);
   const int u = blockIdx.x;
   const int n = len[u / units_per_seq];
   if (n < 0 || n > cap) {
     if (threadIdx.x == 0 && u % units_per_seq == 0) vd::record_status(status, vd::kStDeviceLen);
     return;
   }
-  hi[threadIdx.x] = 0.f;
-  lo[threadIdx.x] = 0.f;
-  __syncthreads();
   const uint16_t* vb = v + (size_t)u * cap * d;
-  vd::accumulate_rows(vb, d, 0, d >> 3, lpr, n,
-                      [&](int i, int& row, float& sign) { row = i; sign = 1.f; }, hi, lo);
+  vd::sum_rows(vb, d, 0, d >> 3, lpr, n, [](int i) { return i; }, [](int) { return 1.f; }, S,
+               ring);
   if ((int)threadIdx.x < d)
-    rs[(size_t)u * d + threadIdx.x] = (double)hi[threadIdx.x] + (double)lo[threadIdx.x];
+    rs[(size_t)u * d + threadIdx.x] = (double)S.acc_hi[threadIdx.x] + (double)S.acc_lo[threadIdx.x];
 }
 
 // ---------------------------------------------------------------------------
@@ -194,30 +194,46 @@ bool cluster_fits(const void* kern, long long units, int c, size_t smem) {
   return ncl > 0;
 }
 
-// CTAs per unit: enough CTAs to cover the GPU several times over, while each
-// CTA still moves row segments of at least 64 bytes of [K | V].  The
-// environment variable VD_CLUSTER_SIZE (1, 2, 4, 8 or 16) overrides the
-// choice, for tuning.
-int choose_cluster(const void* kern, long long units, int d, size_t smem, const DeviceState& st) {
+bool cluster_allowed(int c, int d) {
   const int total_chunks = 2 * (d / 8);
-  int max_c = 1;
-  for (int c = 2; c <= 16; c *= 2)
-    if (total_chunks % c == 0 && total_chunks / c >= 4) max_c = c;
-  int c = 1;
+  return c == 1 || (total_chunks % c == 0 && total_chunks / c >= 4);
+}
+
+// CTAs per unit.  Every candidate C in {1, 2, 4, 8, 16} that keeps row
+// segments of at least 64 bytes of [K | V] is scored by how well its CTAs
+// fill whole waves of the GPU (resident CTAs per SM from the occupancy
+// calculator at that C's shared-memory size); larger clusters pay a small
+// penalty for their per-unit synchronisation.  VD_CLUSTER_SIZE (1, 2, 4, 8
+// or 16) overrides the choice, for tuning.
+int choose_cluster(const void* kern, long long units, int d, int capacity, bool with_select,
+                   const DeviceState& st, size_t* smem_out) {
   const char* env = std::getenv("VD_CLUSTER_SIZE");
   const int want = env ? std::atoi(env) : 0;
-  if (want >= 1 && want <= 16 && (want & (want - 1)) == 0 && total_chunks % want == 0) {
-    c = want;
-  } else {
+  int best_c = 1;
+  double best_score = -1.0;
+  for (int c = 1; c <= 16; c *= 2) {
+    if (want >= 1 && c != want) continue;
+    if (want < 1 && !cluster_allowed(c, d)) continue;
+    if ((d / 8 * 2) % c) continue;
+    const size_t smem = vd::smem_layout(capacity, c, with_select).total;
+    if (smem > (size_t)st.smem_optin) continue;
     int occ = 0;
-    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, kern, kThreads, smem) != cudaSuccess)
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, kern, kThreads, smem) != cudaSuccess) {
       cudaGetLastError();
-    if (occ < 1) occ = 1;
-    const long long slots = (long long)st.sms * occ;
-    while (c < max_c && units * c < 4 * slots) c <<= 1;
+      continue;
+    }
+    if (occ < 1 || !cluster_fits(kern, units, c, smem)) continue;
+    const double slots = (double)st.sms * occ;
+    const double waves = (double)(units * c) / slots;
+    const double eff = waves <= 1.0 ? waves : waves / std::ceil(waves);
+    const double score = eff - 0.02 * std::log2((double)c);
+    if (score > best_score) {
+      best_score = score;
+      best_c = c;
+    }
   }
-  while (c > 1 && !cluster_fits(kern, units, c, smem)) c >>= 1;
-  return c;
+  *smem_out = vd::smem_layout(capacity, best_c, with_select).total;
+  return best_c;
 }
 
 vd_status launch(const void* kern, long long units, int c, size_t smem, const vd::EvictArgs& a,
@@ -242,12 +258,6 @@ vd_status launch(const void* kern, long long units, int c, size_t smem, const vd
   return VD_OK;
 }
 
-size_t evict_smem(int capacity, bool decode) {
-  size_t b = sizeof(vd::Smem);
-  if (!decode) b += (size_t)capacity * 8;
-  return (b + 15) & ~(size_t)15;
-}
-
 vd_status run(const vd_cache* c, int32_t N, const int32_t* N_dev, int32_t B, vd_variant var,
               vd_mu_mode mu, double* running_sum, int32_t* evicted_out, int32_t* kept_idx_out,
               float* scores_out, cudaStream_t s, bool decode, bool score_only) {
@@ -268,8 +278,9 @@ vd_status run(const vd_cache* c, int32_t N, const int32_t* N_dev, int32_t B, vd_
 
   // score-only uses the decode instantiation: it needs no per-token buffers
   const bool small = decode || score_only;
-  const size_t smem = evict_smem(c->capacity, small);
-  if (smem > (size_t)st->smem_optin) return VD_ERR_UNSUPPORTED;
+  if (!small && c->capacity > 65536) return VD_ERR_UNSUPPORTED;  // 16-bit slot lists
+  if (vd::smem_layout(c->capacity, 16, !small).total > (size_t)st->smem_optin)
+    return VD_ERR_UNSUPPORTED;
   const void* kern = evict_kernel(var, small);
   const long long units = (long long)c->n_seq * c->n_layer * c->n_kv_head;
 
@@ -291,7 +302,9 @@ vd_status run(const vd_cache* c, int32_t N, const int32_t* N_dev, int32_t B, vd_
   a.B = decode ? 1 : B;
   a.mu_running = (!score_only && mu == VD_MU_RUNNING) ? 1 : 0;
   a.score_only = score_only ? 1 : 0;
-  a.cluster = choose_cluster(kern, units, c->head_dim, smem, *st);
+  size_t smem = 0;
+  a.cluster = choose_cluster(kern, units, c->head_dim, c->capacity, !small, *st, &smem);
+  if (smem > (size_t)st->smem_optin) return VD_ERR_UNSUPPORTED;
 
   r = launch(kern, units, a.cluster, smem, a, s);
   if (r != VD_OK || score_only) return r;
@@ -361,7 +374,8 @@ vd_status vd_running_sum_init(const vd_cache* c, double* running_sum, vd_stream_
   r = device_state(&st);
   if (r != VD_OK) return r;
   const long long units = (long long)c->n_seq * c->n_layer * c->n_kv_head;
-  vd_rsum_init_kernel<<<(unsigned)units, kThreads, 0, reinterpret_cast<cudaStream_t>(stream)>>>(
+  const size_t smem = vd::smem_layout(c->capacity, 1, false).total;
+  vd_rsum_init_kernel<<<(unsigned)units, kThreads, smem, reinterpret_cast<cudaStream_t>(stream)>>>(
       static_cast<const uint16_t*>(c->v), c->len, running_sum, c->n_layer * c->n_kv_head,
       c->capacity, c->head_dim, lanes_per_row(c->head_dim), st->status);
   if (cudaGetLastError() != cudaSuccess) return VD_ERR_CUDA;

@@ -1,5 +1,6 @@
 // vd_device.cuh -- device-side building blocks of the GB300 (sm_103a) ValueDiff
-// eviction kernels: bf16 unpacking, compensated fp32 sums, thread-block
+// eviction kernels: bf16 unpacking, asynchronous copies, double-float sums,
+// thread-block
 // cluster primitives (distributed shared memory, hardware cluster barrier) and
 // block-wide scans/reductions for a 256-thread CTA.
 #pragma once
@@ -44,6 +45,34 @@ __device__ __forceinline__ uint4 ld_cg16(const void* p) {
                : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w)
                : "l"(p));
   return r;
+}
+
+// Asynchronous 16-byte global -> shared copy (LDGSTS), bypassing L1 and the
+// register file; completion is tracked per thread with commit/wait groups.
+__device__ __forceinline__ void cp_async16(uint32_t smem, const void* gptr) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem), "l"(gptr) : "memory");
+}
+
+__device__ __forceinline__ void cp_async_commit() {
+  asm volatile("cp.async.commit_group;" ::: "memory");
+}
+
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+}
+
+__device__ __forceinline__ uint4 ld_shared16(uint32_t addr) {
+  uint4 r;
+  asm volatile("ld.shared.v4.u32 {%0,%1,%2,%3}, [%4];"
+               : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w)
+               : "r"(addr)
+               : "memory");
+  return r;
+}
+
+__device__ __forceinline__ void st_cluster_u16(uint32_t addr, uint16_t v) {
+  asm volatile("st.shared::cluster.u16 [%0], %1;" ::"r"(addr), "h"(v) : "memory");
 }
 
 __device__ __forceinline__ void st16(void* p, const uint4& v) {

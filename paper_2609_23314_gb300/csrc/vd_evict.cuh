@@ -1,34 +1,41 @@
 // vd_evict.cuh -- the fused ValueDiff eviction kernel for GB300 (sm_103a).
 //
 // One thread-block cluster of C CTAs owns one (sequence, layer, KV head) unit
-// and runs pi_N of Sec. 2.1, Eq. (eviction) on it in a single launch:
+// and runs pi_N of Sec. 2.1, Eq. (eviction) on it in a single launch.  CTA r
+// of the cluster scores the rows [r*R, (r+1)*R) (R = ceil(n / C)) and moves
+// the column slice r of the concatenated [K | V] row.
 //
-//   1. mean   mean = (1/n) sum_i v_i (Sec. 3.2, Eq. vd).  Each CTA sums its
-//             row range as double-float (hi + lo) fp32 pairs per column, and the cluster adds the C partials
-//             in rank order through distributed shared memory, so every CTA
+//   1. mean   mean = (1/n) sum_i v_i (Sec. 3.2, Eq. vd) as double-float
+//             (hi + lo) fp32 column sums; the C partials are added in rank
+//             order through distributed shared memory (DSMEM), so every CTA
 //             holds the same mean.  Running-sum mode adds only the appended
-//             rows to the caller's fp64 sum S.
-//   2. score  16-byte bf16 loads, d/8 lanes per row, warp-shuffle reduction
-//             of the row's squared deviation (L2), its norm (Norm) or its
-//             normalised difference (Dir, as 1/2 |v/|v| - mean/|mean||^2,
-//             which equals 1 - cos without cancellation).
-//   3. select block prompt processing (N+B -> N): every CTA receives all n
-//             fp32 scores (as order-preserving uint32 keys) through DSMEM
-//             and runs a 4-pass 8-bit radix select for the N-th largest key t;
-//             keys > t are kept and the keys == t with the lowest slot
-//             indices fill the rest.  Decode (N+1 -> N): a cluster arg-min
-//             over (key, -index) finds the one evicted slot.
-//   4. list   block prefix sums turn the keep flags into perm: the kept slots
-//             ascending in perm[0, N), the evicted ones after them.
-//   5. sum    running-sum mode: S += sum(appended rows) - sum(evicted rows),
-//             for the V columns this CTA compacts, before it moves them.
-//   6. move   K' = gather(K, perm), V' = gather(V, perm) in place.  CTA r
-//             owns a disjoint column slice of [K | V] and walks the rows
-//             r = first evicted .. N-1 upward in register tiles: a tile's
-//             sources are all loaded before any of its destinations is
-//             stored (one __syncthreads), and the next tile's loads are
-//             issued before this tile's stores.  Because perm[r] >= r, a
-//             store never hits a row a later tile still has to read.
+//             rows (spread over the cluster) to the caller's fp64 sum S.
+//   2. score  rows stream through a per-thread ring of asynchronous 16-byte
+//             copies (cp.async, 4 stages in flight); d/8 lanes per row, warp
+//             shuffle reduction of the squared deviation (L2), of the norm
+//             (Norm), or of the normalised difference (Dir, as
+//             1/2 |v/|v| - mean/|mean||^2, which equals 1 - cos without
+//             cancellation).  Scores become order-preserving uint32 keys.
+//   3. select block prompt processing (N+B -> N): a 4-pass 8-bit radix select
+//             for the N-th largest key t; every CTA histograms only its own
+//             rows and the cluster adds the C histograms through DSMEM.
+//             Keys > t are kept, and the keys == t with the lowest slots fill
+//             the rest (the lower-index tie-break).  Decode (N+1 -> N): a
+//             cluster arg-min over (key, -slot) finds the one evicted slot.
+//   4. list   per-CTA counts (> t, == t) are exchanged, each CTA ranks its own
+//             rows with block prefix sums and scatters them into every CTA's
+//             perm[] (uint16): kept slots ascending in [0, N), then the
+//             evicted slots ascending.
+//   5. sum    running-sum mode: S += sum(appended rows) - sum(evicted rows)
+//             over the V columns this CTA moves, before it moves them.
+//   6. move   K' = gather(K, perm), V' = gather(V, perm), in place, for the
+//             rows r = first evicted .. N-1 of this CTA's column slice.  Tiles
+//             of rows stream through the cp.async ring; tile t is stored only
+//             after every thread's copies of tile t have landed (one
+//             __syncthreads), while tiles t+1.. are already in flight.  Since
+//             perm[r] >= r, a tile's destinations lie below every source a
+//             later tile reads, so the ascending order is hazard-free, and
+//             column slices make the CTAs of a unit independent.
 //
 // Nothing waits on a flag; the only cross-CTA synchronisation is the hardware
 // cluster barrier, which every CTA of a cluster reaches the same number of
@@ -42,6 +49,11 @@
 #include "vd_device.cuh"
 
 namespace vd {
+
+// cp.async ring: kRingStages stages of kRingItems 16-byte copies per thread.
+constexpr int kRingStages = 4;
+constexpr int kRingItems = 2;
+constexpr int kRingBytes = kRingStages * kRingItems * kThreads * 16;
 
 struct EvictArgs {
   uint16_t* k;            // bf16 [U][capacity][d]
@@ -64,71 +76,101 @@ struct EvictArgs {
   int32_t cluster;        // C, CTAs per unit
 };
 
-// Fixed part of the dynamic shared memory; the general (block) kernel appends
-// keys[capacity] and perm[capacity].
+// Fixed part of the dynamic shared memory.  After it (16-byte aligned): the
+// cp.async ring, then (block eviction only) this CTA's keys [R] and the
+// unit's perm [capacity] (uint16).
 struct Smem {
   float mu[256];
   float muhat[256];
   float acc_hi[256];  // this CTA's partial column sums (read by peer CTAs)
   float acc_lo[256];
-  uint32_t hist[256];
+  uint32_t hist[2][256];  // this CTA's radix histograms (read by peers)
+  uint32_t ghist[256];
   int scan[kWarps];
   float fsh[kWarps];
-  unsigned long long best;  // decode: this CTA's (key, -index) minimum
+  unsigned long long best;  // decode: this CTA's (key, -slot) minimum
   unsigned long long wbest[kWarps];
   int sel_digit, sel_above, sel_cnt;
-  int e_first;
+  int cnt_gt, cnt_eq;  // this CTA's keys > t and == t (read by peers)
   int mu_zero;
 };
 
-// Sums rows of one unit's V, restricted to 16-byte column chunks
-// [chunk0, chunk0 + nchunks), into acc_hi/acc_lo (which the caller zeroed).
-// Item i contributes sign(i) * V[row(i)].  Lanes are grouped P per row
-// (P = power of two >= nchunks); partials merge across the warp with TwoSum
-// shuffles and across warps in a fixed order, so the result is deterministic.
-template <class RowOf>
-__device__ __forceinline__ void accumulate_rows(const uint16_t* __restrict__ vbase, int d,
-                                                int chunk0, int nchunks, int P, int count,
-                                                RowOf row_of, float* acc_hi, float* acc_lo) {
-  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+__host__ __device__ constexpr size_t align16(size_t x) { return (x + 15) & ~(size_t)15; }
+
+// Byte offsets of the variable parts; the host sizes the launch with the same
+// function.
+struct SmemLayout {
+  size_t ring, keys, perm, total;
+};
+
+__host__ __device__ inline SmemLayout smem_layout(int capacity, int cluster, bool with_select) {
+  SmemLayout l;
+  l.ring = align16(sizeof(Smem));
+  l.keys = l.ring + kRingBytes;
+  const size_t rows = with_select ? (size_t)((capacity + cluster - 1) / cluster) : 0;
+  l.perm = l.keys + align16(rows * 4);
+  l.total = l.perm + (with_select ? align16((size_t)capacity * 2) : 0);
+  return l;
+}
+
+// Streams items [0, count) through a thread-private cp.async ring.  Item i is
+// row row_of(i) of `base` (row stride d elements); in every group of P lanes
+// (P a power of two >= nchunks) lane ci copies 16-byte chunk chunk0 + ci.
+// Thread group g takes items g, g + ng, g + 2 ng, ...  All threads run the
+// same number of steps, so consume() may use warp shuffles; it receives every
+// item slot with `in` = item < count and the chunk (zeros for idle lanes).
+// A thread only reuses a ring slot after its own consume() used the data.
+template <class RowOf, class Consume>
+__device__ __forceinline__ void stream_rows(const uint16_t* __restrict__ base, int d, int chunk0,
+                                            int nchunks, int P, int count, RowOf row_of,
+                                            Consume consume, uint32_t ring) {
+  const int tid = threadIdx.x, lane = tid & 31;
   const int ci = lane & (P - 1);
   const bool active = ci < nchunks;
-  const int ng = kThreads / P;
-  const int g = tid / P;
-  const int col = (chunk0 + ci) * 8;
-  float s[8], c[8];
+  const int ng = kThreads / P, g = tid / P;
+  const int per_stage = ng * kRingItems;
+  const int nst = count > 0 ? (count + per_stage - 1) / per_stage : 0;
+  const uint32_t my = ring + (uint32_t)tid * 16u;
+  const uint16_t* colp = base + (chunk0 + ci) * 8;
+  auto slot = [&](int s, int u) {
+    return my + (uint32_t)((s * kRingItems + u) * kThreads * 16);
+  };
+  auto issue = [&](int st) {
+    if (st < nst) {
 #pragma unroll
-  for (int k = 0; k < 8; ++k) s[k] = c[k] = 0.f;
-  constexpr int U = 4;
-  for (int base = g; base < count; base += ng * U) {
-    uint4 q[U];
-    float sg[U];
-#pragma unroll
-    for (int i = 0; i < U; ++i) {
-      const int it = base + i * ng;
-      q[i] = make_uint4(0, 0, 0, 0);
-      sg[i] = 0.f;
-      if (active && it < count) {
-        int row;
-        float sign;
-        row_of(it, row, sign);
-        q[i] = ld_cg16(vbase + (size_t)row * d + col);
-        sg[i] = sign;
+      for (int u = 0; u < kRingItems; ++u) {
+        const int item = g + (st * kRingItems + u) * ng;
+        if (active && item < count)
+          cp_async16(slot(st % kRingStages, u), colp + (size_t)row_of(item) * d);
       }
     }
+    cp_async_commit();
+  };
+  for (int st = 0; st < kRingStages; ++st) issue(st);
+  for (int st = 0; st < nst; ++st) {
+    cp_async_wait<kRingStages - 1>();
 #pragma unroll
-    for (int i = 0; i < U; ++i) {
-      if (sg[i] != 0.f) {
-        float x[8];
-        unpack8(q[i], x);
-#pragma unroll
-        for (int k = 0; k < 8; ++k) ff_accumulate(s[k], c[k], sg[i] * x[k]);
-      }
+    for (int u = 0; u < kRingItems; ++u) {
+      const int item = g + (st * kRingItems + u) * ng;
+      const bool in = item < count;
+      uint4 q = make_uint4(0, 0, 0, 0);
+      if (active && in) q = ld_shared16(slot(st % kRingStages, u));
+      consume(item, in, q);
     }
+    issue(st + kRingStages);
   }
+  cp_async_wait<0>();
+}
+
+// Merges every thread's double-float column partials (8 columns from column
+// `col`, lanes grouped P per row) into acc_hi/acc_lo (zeroed by the caller),
+// across the warp with TwoSum shuffles and across warps in a fixed order.
+__device__ __forceinline__ void merge_columns(float (&hi)[8], float (&lo)[8], int P, bool active,
+                                              int col, float* acc_hi, float* acc_lo) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   ff p[8];
 #pragma unroll
-  for (int k = 0; k < 8; ++k) p[k] = ff_add(ff{s[k], 0.f}, ff{0.f, c[k]});
+  for (int k = 0; k < 8; ++k) p[k] = ff_add(ff{hi[k], 0.f}, ff{0.f, lo[k]});
   for (int off = P; off < 32; off <<= 1) {
 #pragma unroll
     for (int k = 0; k < 8; ++k) p[k] = ff_add(p[k], ff_shfl_xor(p[k], off));
@@ -146,10 +188,32 @@ __device__ __forceinline__ void accumulate_rows(const uint16_t* __restrict__ vba
   }
 }
 
-__device__ __forceinline__ void zero_acc(Smem& S) {
+// acc (zeroed here) <- sum over items [0, count) of sign(item) * V[row(item)],
+// restricted to 16-byte column chunks [chunk0, chunk0 + nchunks).
+template <class RowOf, class SignOf>
+__device__ __forceinline__ void sum_rows(const uint16_t* vbase, int d, int chunk0, int nchunks,
+                                         int P, int count, RowOf row_of, SignOf sign_of, Smem& S,
+                                         uint32_t ring) {
   S.acc_hi[threadIdx.x] = 0.f;
   S.acc_lo[threadIdx.x] = 0.f;
   __syncthreads();
+  const int ci = (threadIdx.x & 31) & (P - 1);
+  const bool active = ci < nchunks;
+  float hi[8], lo[8];
+#pragma unroll
+  for (int k = 0; k < 8; ++k) hi[k] = lo[k] = 0.f;
+  stream_rows(vbase, d, chunk0, nchunks, P, count, row_of,
+              [&](int item, bool in, const uint4& q) {
+                if (in && active) {
+                  float x[8];
+                  unpack8(q, x);
+                  const float sg = sign_of(item);
+#pragma unroll
+                  for (int k = 0; k < 8; ++k) ff_accumulate(hi[k], lo[k], sg * x[k]);
+                }
+              },
+              ring);
+  merge_columns(hi, lo, P, active, (chunk0 + ci) * 8, S.acc_hi, S.acc_lo);
 }
 
 // Order-preserving key of a non-negative score; NaN ranks lowest.  `bad`
@@ -159,32 +223,46 @@ __device__ __forceinline__ uint32_t score_key(float s, bool& bad) {
   return (s == s) ? __float_as_uint(s) : 0u;
 }
 
-// Radix select over keys[0, n): t = the N-th largest key (1-based), keep_eq =
-// how many keys equal to t survive, cnt_eq = how many keys equal t.
+// Radix select over the keys of the whole cluster: t = the N-th largest key
+// (1-based), keep_eq = how many keys equal to t survive, cnt_eq = how many
+// keys equal t.  `keys` holds this CTA's R keys.
 struct Selection {
   uint32_t t;
   int keep_eq;
   int cnt_eq;
 };
 
-__device__ __forceinline__ Selection radix_select(const uint32_t* keys, int n, int N, Smem& S) {
+__device__ __forceinline__ Selection cluster_radix_select(const uint32_t* keys, int R, int N,
+                                                          int C, Smem& S) {
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   uint32_t prefix = 0, pmask = 0;
-  int need = N, cnt = n;
+  int need = N, cnt = 0;
   for (int pass = 0; pass < 4; ++pass) {
     const int shift = 24 - 8 * pass;
-    S.hist[tid] = 0;
+    uint32_t* h = S.hist[pass & 1];
+    h[tid] = 0;
     __syncthreads();
-    for (int base = 0; base < n; base += kThreads) {
+    for (int base = 0; base < R; base += kThreads) {
       const int j = base + tid;
-      const uint32_t key = j < n ? keys[j] : 0u;
-      const bool match = j < n && (key & pmask) == prefix;
+      const uint32_t key = j < R ? keys[j] : 0u;
+      const bool match = j < R && (key & pmask) == prefix;
       const unsigned act = __ballot_sync(kFull, match);
       if (match) {
         const uint32_t dig = (key >> shift) & 255u;
         const unsigned peers = __match_any_sync(act, dig);
-        if (lane == __ffs(peers) - 1) atomicAdd(&S.hist[dig], (uint32_t)__popc(peers));
+        if (lane == __ffs(peers) - 1) atomicAdd(&h[dig], (uint32_t)__popc(peers));
       }
+    }
+    if (C > 1) cluster_sync(); else __syncthreads();
+    {
+      uint32_t tot = 0;
+      if (C > 1) {
+        const uint32_t a = smem_addr(&h[tid]);
+        for (int rr = 0; rr < C; ++rr) tot += ld_cluster_u32(mapa(a, (unsigned)rr));
+      } else {
+        tot = h[tid];
+      }
+      S.ghist[tid] = tot;
     }
     __syncthreads();
     if (warp == 0) {
@@ -192,7 +270,7 @@ __device__ __forceinline__ Selection radix_select(const uint32_t* keys, int n, i
       int sum = 0;
 #pragma unroll
       for (int i = 0; i < 8; ++i) {
-        c[i] = (int)S.hist[255 - (lane * 8 + i)];
+        c[i] = (int)S.ghist[255 - (lane * 8 + i)];
         sum += c[i];
       }
       int incl = sum;
@@ -225,109 +303,120 @@ __device__ __forceinline__ Selection radix_select(const uint32_t* keys, int n, i
   return {prefix, need, cnt};
 }
 
-// Keep flags -> perm (kept slots ascending, then evicted slots ascending) and
-// the first evicted slot.  Threads own contiguous index chunks so the prefix
-// sums follow slot order, which is what gives ties to the lower index.
-__device__ __forceinline__ void build_perm(const uint32_t* keys, int n, int N, Selection sel, int* perm,
-                           Smem& S) {
+// Ranks this CTA's rows [r0, r0 + R) against the selection and scatters them
+// into perm[] of every CTA of the cluster: kept slots ascending at [0, N),
+// evicted slots ascending at [N, n).  Threads own contiguous row chunks, so
+// prefix sums follow slot order (ties go to the lower slot).  Ends with the
+// cluster barrier after which every CTA's perm[] is complete.
+__device__ __forceinline__ void cluster_build_perm(const uint32_t* keys, int r0, int R, int N,
+                                                   Selection sel, int C, unsigned rank,
+                                                   uint16_t* perm, Smem& S) {
   const int tid = threadIdx.x;
-  const int ch = (n + kThreads - 1) / kThreads;
-  const int c0 = min(n, tid * ch), c1 = min(n, c0 + ch);
+  const int ch = (R + kThreads - 1) / kThreads;
+  const int c0 = min(R, tid * ch), c1 = min(R, c0 + ch);
   const uint32_t t = sel.t;
-  const bool scan_ties = sel.cnt_eq > sel.keep_eq;
-  const int q = scan_ties ? sel.keep_eq : INT_MAX;
-  int total;
-  int tie_ex = 0;
-  if (scan_ties) {
-    int nt = 0;
-    for (int j = c0; j < c1; ++j) nt += keys[j] == t;
-    tie_ex = block_exclusive_scan(nt, S.scan, total);
+  int ngt = 0, neq = 0;
+  for (int j = c0; j < c1; ++j) {
+    ngt += keys[j] > t;
+    neq += keys[j] == t;
   }
-  int nk = 0;
-  {
-    int tr = tie_ex;
-    for (int j = c0; j < c1; ++j) {
-      const uint32_t key = keys[j];
-      const bool eq = key == t;
-      nk += (key > t) || (eq && tr < q);
-      tr += eq;
-    }
+  int tot_gt, tot_eq;
+  const int gt_ex = block_exclusive_scan(ngt, S.scan, tot_gt);
+  const int eq_ex = block_exclusive_scan(neq, S.scan, tot_eq);
+  if (tid == 0) {
+    S.cnt_gt = tot_gt;
+    S.cnt_eq = tot_eq;
   }
-  if (tid == 0) S.e_first = INT_MAX;
-  const int kept_ex = block_exclusive_scan(nk, S.scan, total);
-  int kp = kept_ex, tr = tie_ex, ef = INT_MAX;
+  if (C > 1) cluster_sync(); else __syncthreads();
+  // ties and kept rows of the lower-ranked CTAs
+  const int q = sel.keep_eq;
+  int tie_off = 0, kept_off = 0;
+  for (int rr = 0; rr < (int)rank; ++rr) {
+    const int g = (int)ld_cluster_u32(mapa(smem_addr(&S.cnt_gt), rr));
+    const int e = (int)ld_cluster_u32(mapa(smem_addr(&S.cnt_eq), rr));
+    kept_off += g + min(max(q - tie_off, 0), e);
+    tie_off += e;
+  }
+  const int my_tie_quota = max(q - tie_off, 0);  // ties this CTA may still keep
+  int tie_rank = eq_ex;                          // ties of this CTA before the chunk
+  int kp = kept_off + gt_ex + min(my_tie_quota, eq_ex);
+  const uint32_t perm_addr = smem_addr(perm);
   for (int j = c0; j < c1; ++j) {
     const uint32_t key = keys[j];
     const bool eq = key == t;
-    const bool keep = (key > t) || (eq && tr < q);
-    tr += eq;
-    if (keep) {
-      perm[kp++] = j;
+    const bool keep = key > t || (eq && tie_rank < my_tie_quota);
+    tie_rank += eq;
+    const int row = r0 + j;
+    const int pos = keep ? kp : N + (row - kp);
+    kp += keep;
+    if (C > 1) {
+      for (int cc = 0; cc < C; ++cc)
+        st_cluster_u16(mapa(perm_addr + 2u * (unsigned)pos, (unsigned)cc), (uint16_t)row);
     } else {
-      perm[N + (j - kp)] = j;
-      ef = min(ef, j);
+      perm[pos] = (uint16_t)row;
     }
   }
-  if (ef != INT_MAX) atomicMin(&S.e_first, ef);
-  __syncthreads();
+  if (C > 1) cluster_sync(); else __syncthreads();
 }
 
 // In-place, order-preserving move of rows [r_begin, r_end) of the column
 // slice [chunk0, chunk0 + cps) of the concatenated [K | V] row: row r takes
 // source row perm[r] (or r + 1 when perm is null: the decode shift).
-template <int UC>
 __device__ __forceinline__ void compact_slice(uint16_t* kb, uint16_t* vb, int d, int chunk0,
                                               int cps, int r_begin, int r_end,
-                                              const int* perm) {
+                                              const uint16_t* perm, uint32_t ring) {
+  const int tid = threadIdx.x;
   const int d8 = d >> 3;
   const int rs = kThreads / cps;
-  const bool on = (int)threadIdx.x < rs * cps;
-  const int my_ch = chunk0 + (int)threadIdx.x % cps;
-  const int my_off = (int)threadIdx.x / cps;
+  const bool on = tid < rs * cps;
+  const int my_ch = chunk0 + tid % cps;
+  const int my_off = tid / cps;
   uint16_t* col = my_ch < d8 ? kb + my_ch * 8 : vb + (my_ch - d8) * 8;
-  const int tile = rs * UC;
+  const int tile = rs * kRingItems;
   const int ntiles = r_end > r_begin ? (r_end - r_begin + tile - 1) / tile : 0;
-  uint4 A[UC], Bq[UC];
-
-  auto load = [&](uint4 (&X)[UC], int t) {
+  const uint32_t my = ring + (uint32_t)tid * 16u;
+  auto slot = [&](int s, int u) {
+    return my + (uint32_t)((s * kRingItems + u) * kThreads * 16);
+  };
+  auto issue = [&](int t) {
+    if (t < ntiles) {
 #pragma unroll
-    for (int i = 0; i < UC; ++i) {
-      const int r = r_begin + t * tile + i * rs + my_off;
-      if (on && r < r_end) {
-        const int src = perm ? perm[r] : r + 1;
-        X[i] = ld_cg16(col + (size_t)src * d);
+      for (int u = 0; u < kRingItems; ++u) {
+        const int r = r_begin + t * tile + u * rs + my_off;
+        if (on && r < r_end) {
+          const int src = perm ? (int)perm[r] : r + 1;
+          cp_async16(slot(t % kRingStages, u), col + (size_t)src * d);
+        }
       }
     }
+    cp_async_commit();
   };
-  auto store = [&](const uint4 (&X)[UC], int t) {
+  for (int t = 0; t < kRingStages; ++t) issue(t);
+  for (int t = 0; t < ntiles; ++t) {
+    cp_async_wait<kRingStages - 1>();
+    __syncthreads();  // every source of tile t is in shared memory
 #pragma unroll
-    for (int i = 0; i < UC; ++i) {
-      const int r = r_begin + t * tile + i * rs + my_off;
-      if (on && r < r_end) st16(col + (size_t)r * d, X[i]);
+    for (int u = 0; u < kRingItems; ++u) {
+      const int r = r_begin + t * tile + u * rs + my_off;
+      if (on && r < r_end) st16(col + (size_t)r * d, ld_shared16(slot(t % kRingStages, u)));
     }
-  };
-
-  if (ntiles > 0) load(A, 0);
-  for (int t = 0; t < ntiles; t += 2) {
-    __syncthreads();  // every source of tile t has been loaded
-    if (t + 1 < ntiles) load(Bq, t + 1);
-    store(A, t);
-    if (t + 1 >= ntiles) break;
-    __syncthreads();  // every source of tile t + 1 has been loaded
-    if (t + 2 < ntiles) load(A, t + 2);
-    store(Bq, t + 1);
+    issue(t + kRingStages);
   }
+  cp_async_wait<0>();
 }
 
 template <int VAR, bool DECODE>
-__global__ void __launch_bounds__(kThreads, 4) evict_kernel(const EvictArgs a) {
+__global__ void __launch_bounds__(kThreads, DECODE ? 4 : 3) evict_kernel(const EvictArgs a) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   Smem& S = *reinterpret_cast<Smem*>(smem_raw);
-  uint32_t* keys = reinterpret_cast<uint32_t*>(smem_raw + sizeof(Smem));
-  int* perm = reinterpret_cast<int*>(keys + a.capacity);
+  const int C = a.cluster;
+  const bool with_select = !DECODE && !a.score_only;
+  const SmemLayout L = smem_layout(a.capacity, C, with_select);
+  const uint32_t ring = smem_addr(smem_raw + L.ring);
+  uint32_t* keys = reinterpret_cast<uint32_t*>(smem_raw + L.keys);
+  uint16_t* perm = reinterpret_cast<uint16_t*>(smem_raw + L.perm);
 
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  const int C = a.cluster;
   const unsigned rank = C > 1 ? cluster_ctarank() : 0u;
   const int u = C > 1 ? (int)cluster_id_x() : (int)blockIdx.x;
   const int d = a.d, d8 = d >> 3;
@@ -361,6 +450,7 @@ __global__ void __launch_bounds__(kThreads, 4) evict_kernel(const EvictArgs a) {
   const int vchunks = max(0, chunk0 + cps - max(chunk0, d8));
   int vp = 1;
   while (vp < vchunks) vp <<= 1;
+  const int first_new = n - a.B;
 
   if (!evict && !a.score_only) {
     // ---- nothing to evict: identity outputs, running sum += appended rows ---
@@ -369,11 +459,8 @@ __global__ void __launch_bounds__(kThreads, 4) evict_kernel(const EvictArgs a) {
         a.kept_out[(size_t)u * a.N + i] = i < n ? i : -1;
     if (DECODE && a.evicted_out && rank == 0 && tid == 0) a.evicted_out[u] = -1;
     if (a.mu_running && a.B > 0 && vchunks > 0) {
-      zero_acc(S);
-      const int first_new = n - a.B;
-      accumulate_rows(vb, d, vchunk0, vchunks, vp, a.B,
-                      [&](int i, int& row, float& sign) { row = first_new + i; sign = 1.f; },
-                      S.acc_hi, S.acc_lo);
+      sum_rows(vb, d, vchunk0, vchunks, vp, a.B, [&](int i) { return first_new + i; },
+               [](int) { return 1.f; }, S, ring);
       if (tid < vchunks * 8) {
         const int c = vchunk0 * 8 + tid;
         double* sp = a.running_sum + (size_t)u * d + c;
@@ -389,11 +476,17 @@ __global__ void __launch_bounds__(kThreads, 4) evict_kernel(const EvictArgs a) {
   const int lpr = a.lpr;
   if (VAR != 2) {
     const bool run = a.mu_running && !a.score_only;
-    const int p0 = run ? max(r0, n - a.B) : r0;
-    zero_acc(S);
-    accumulate_rows(vb, d, 0, d8, lpr, max(0, r1 - p0),
-                    [&](int i, int& row, float& sign) { row = p0 + i; sign = 1.f; },
-                    S.acc_hi, S.acc_lo);
+    int p0, p1;
+    if (run) {  // the appended rows, spread over the cluster
+      const int per = (a.B + C - 1) / C;
+      p0 = min(n, first_new + (int)rank * per);
+      p1 = min(n, p0 + per);
+    } else {
+      p0 = r0;
+      p1 = r1;
+    }
+    sum_rows(vb, d, 0, d8, lpr, max(0, p1 - p0), [&](int i) { return p0 + i; },
+             [](int) { return 1.f; }, S, ring);
     if (C > 1) cluster_sync(); else __syncthreads();
     if (tid < d) {
       ff t{0.f, 0.f};
@@ -420,16 +513,15 @@ __global__ void __launch_bounds__(kThreads, 4) evict_kernel(const EvictArgs a) {
       __syncthreads();
     }
   }
-  // score-only and decode read peer shared memory below or above; release
-  // the cluster barrier phase once the last peer access is done
-  const bool split_exit = C > 1 && (a.score_only || DECODE) && VAR != 2;
+  // vd_score reads peer partial sums above and nothing after: release that
+  // barrier phase now, wait for it before exiting (peers may still be reading)
+  const bool score_split = C > 1 && a.score_only && VAR != 2;
+  if (score_split) cluster_arrive();
 
   // ---- 2. scores -------------------------------------------------------
   {
     const int ci = lane & (lpr - 1);
     const bool active = ci < d8;
-    const int ng = kThreads / lpr;
-    const int g = tid / lpr;
     float m8[8], h8[8];
 #pragma unroll
     for (int k = 0; k < 8; ++k) {
@@ -437,79 +529,64 @@ __global__ void __launch_bounds__(kThreads, 4) evict_kernel(const EvictArgs a) {
       h8[k] = (VAR == 1 && active) ? S.muhat[ci * 8 + k] : 0.f;
     }
     const bool mu_zero = VAR == 1 && S.mu_zero;
-    const uint32_t keys_addr = smem_addr(keys);
     unsigned long long best = ~0ull;
     float* sc_out = a.scores_out ? a.scores_out + (size_t)u * a.capacity : nullptr;
-    constexpr int U = 4;
-    // trip count uniform over the CTA: the row reductions below shuffle
-    for (int b0 = r0; b0 < r1; b0 += ng * U) {
-      uint4 q[U];
+    stream_rows(
+        vb, d, 0, d8, lpr, r1 - r0, [&](int i) { return r0 + i; },
+        [&](int item, bool in, const uint4& q) {
+          float x[8];
+          unpack8(q, x);
+          float s;
+          if (VAR == 0) {
+            float acc = 0.f;
 #pragma unroll
-      for (int i = 0; i < U; ++i) {
-        const int r = b0 + g + i * ng;
-        q[i] = (active && r < r1) ? ld_cg16(vb + (size_t)r * d + ci * 8) : make_uint4(0, 0, 0, 0);
-      }
+            for (int k = 0; k < 8; ++k) {
+              const float dv = x[k] - m8[k];
+              acc = fmaf(dv, dv, acc);
+            }
+            for (int off = 1; off < lpr; off <<= 1) acc += __shfl_xor_sync(kFull, acc, off);
+            s = sqrtf(acc);
+          } else if (VAR == 2) {
+            float acc = 0.f;
 #pragma unroll
-      for (int i = 0; i < U; ++i) {
-        const int r = b0 + g + i * ng;
-        float x[8];
-        unpack8(q[i], x);
-        float s;
-        if (VAR == 0) {
-          float acc = 0.f;
+            for (int k = 0; k < 8; ++k) acc = fmaf(x[k], x[k], acc);
+            for (int off = 1; off < lpr; off <<= 1) acc += __shfl_xor_sync(kFull, acc, off);
+            s = sqrtf(acc);
+          } else {
+            float nv = 0.f;
 #pragma unroll
-          for (int k = 0; k < 8; ++k) {
-            const float dv = x[k] - m8[k];
-            acc = fmaf(dv, dv, acc);
+            for (int k = 0; k < 8; ++k) nv = fmaf(x[k], x[k], nv);
+            for (int off = 1; off < lpr; off <<= 1) nv += __shfl_xor_sync(kFull, nv, off);
+            const float inv = nv > 0.f ? 1.f / sqrtf(nv) : 0.f;
+            float acc = 0.f;
+#pragma unroll
+            for (int k = 0; k < 8; ++k) {
+              const float dv = x[k] * inv - h8[k];
+              acc = fmaf(dv, dv, acc);
+            }
+            for (int off = 1; off < lpr; off <<= 1) acc += __shfl_xor_sync(kFull, acc, off);
+            s = (nv > 0.f && !mu_zero) ? 0.5f * acc : 1.f;
           }
-          for (int off = 1; off < lpr; off <<= 1) acc += __shfl_xor_sync(kFull, acc, off);
-          s = sqrtf(acc);
-        } else if (VAR == 2) {
-          float acc = 0.f;
-#pragma unroll
-          for (int k = 0; k < 8; ++k) acc = fmaf(x[k], x[k], acc);
-          for (int off = 1; off < lpr; off <<= 1) acc += __shfl_xor_sync(kFull, acc, off);
-          s = sqrtf(acc);
-        } else {
-          float nv = 0.f;
-#pragma unroll
-          for (int k = 0; k < 8; ++k) nv = fmaf(x[k], x[k], nv);
-          for (int off = 1; off < lpr; off <<= 1) nv += __shfl_xor_sync(kFull, nv, off);
-          const float inv = nv > 0.f ? 1.f / sqrtf(nv) : 0.f;
-          float acc = 0.f;
-#pragma unroll
-          for (int k = 0; k < 8; ++k) {
-            const float dv = x[k] * inv - h8[k];
-            acc = fmaf(dv, dv, acc);
-          }
-          for (int off = 1; off < lpr; off <<= 1) acc += __shfl_xor_sync(kFull, acc, off);
-          s = (nv > 0.f && !mu_zero) ? 0.5f * acc : 1.f;
-        }
-        if (r < r1) {
-          if (ci == 0 && sc_out) sc_out[r] = s;
-          if (!a.score_only) {
-            bool bad;
-            const uint32_t key = score_key(s, bad);
-            if (bad && ci == 0) record_status(a.status, kStNonfinite);
-            if (DECODE) {
-              const unsigned long long pk =
-                  ((unsigned long long)key << 32) | (unsigned long long)(0xffffffffu - (unsigned)r);
-              best = pk < best ? pk : best;
-            } else if (C == 1) {
-              if (ci == 0) keys[r] = key;
-            } else {
-              for (int cc = ci; cc < C; cc += lpr)
-                st_cluster_u32(mapa(keys_addr + 4u * (unsigned)r, (unsigned)cc), key);
+          if (in && ci == 0) {
+            const int r = r0 + item;
+            if (sc_out) sc_out[r] = s;
+            if (!a.score_only) {
+              bool bad;
+              const uint32_t key = score_key(s, bad);
+              if (bad) record_status(a.status, kStNonfinite);
+              if (DECODE) {
+                const unsigned long long pk = ((unsigned long long)key << 32) |
+                                              (unsigned long long)(0xffffffffu - (unsigned)r);
+                best = pk < best ? pk : best;
+              } else {
+                keys[item] = key;
+              }
             }
           }
-        }
-      }
-    }
+        },
+        ring);
     if (a.score_only) {
-      if (split_exit) {
-        cluster_arrive();
-        cluster_wait();
-      }
+      if (score_split) cluster_wait();
       return;
     }
     if (DECODE) {
@@ -523,23 +600,24 @@ __global__ void __launch_bounds__(kThreads, 4) evict_kernel(const EvictArgs a) {
       }
     }
   }
-  if (C > 1) cluster_sync(); else __syncthreads();
 
   // ---- 3./4. select and kept list --------------------------------------
   int e_first;
   if (DECODE) {
+    if (C > 1) cluster_sync(); else __syncthreads();
     unsigned long long b = ~0ull;
     for (int rr = 0; rr < C; ++rr) {
       const unsigned long long o =
           C > 1 ? ld_cluster_u64(mapa(smem_addr(&S.best), rr)) : S.best;
       b = o < b ? o : b;
     }
-    if (split_exit || C > 1) cluster_arrive();  // last peer access of this CTA
+    if (C > 1) cluster_arrive();  // last peer access of this CTA; wait before exit
     e_first = (int)(0xffffffffu - (unsigned)(b & 0xffffffffull));
   } else {
-    const Selection sel = radix_select(keys, n, Nb, S);
-    build_perm(keys, n, Nb, sel, perm, S);
-    e_first = S.e_first;
+    __syncthreads();  // own keys complete
+    const Selection sel = cluster_radix_select(keys, r1 - r0, Nb, C, S);
+    cluster_build_perm(keys, r0, r1 - r0, Nb, sel, C, rank, perm, S);
+    e_first = perm[Nb];
   }
 
   // ---- outputs -----------------------------------------------------------
@@ -547,7 +625,7 @@ __global__ void __launch_bounds__(kThreads, 4) evict_kernel(const EvictArgs a) {
     int32_t* ko = a.kept_out + (size_t)u * a.N;
     for (int i = (int)rank * kThreads + tid; i < a.N; i += C * kThreads) {
       int val = -1;
-      if (i < Nb) val = DECODE ? (i < e_first ? i : i + 1) : perm[i];
+      if (i < Nb) val = DECODE ? (i < e_first ? i : i + 1) : (int)perm[i];
       ko[i] = val;
     }
   }
@@ -555,20 +633,12 @@ __global__ void __launch_bounds__(kThreads, 4) evict_kernel(const EvictArgs a) {
 
   // ---- 5. running sum: S += appended rows - evicted rows (own V columns) --
   if (a.mu_running && vchunks > 0) {
-    zero_acc(S);
-    const int first_new = n - a.B;
-    const int nev = n - Nb;
-    accumulate_rows(vb, d, vchunk0, vchunks, vp, a.B + nev,
-                    [&](int i, int& row, float& sign) {
-                      if (i < a.B) {
-                        row = first_new + i;
-                        sign = 1.f;
-                      } else {
-                        row = DECODE ? e_first : perm[Nb + (i - a.B)];
-                        sign = -1.f;
-                      }
-                    },
-                    S.acc_hi, S.acc_lo);
+    const int B = a.B;
+    sum_rows(vb, d, vchunk0, vchunks, vp, B + (n - Nb),
+             [&](int i) {
+               return i < B ? first_new + i : (DECODE ? e_first : (int)perm[Nb + (i - B)]);
+             },
+             [&](int i) { return i < B ? 1.f : -1.f; }, S, ring);
     if (tid < vchunks * 8) {
       const int c = vchunk0 * 8 + tid;
       double* sp = a.running_sum + (size_t)u * d + c;
@@ -577,7 +647,7 @@ __global__ void __launch_bounds__(kThreads, 4) evict_kernel(const EvictArgs a) {
   }
 
   // ---- 6. in-place compaction of this CTA's column slice ---------------
-  compact_slice<4>(kb, vb, d, chunk0, cps, e_first, Nb, DECODE ? nullptr : perm);
+  compact_slice(kb, vb, d, chunk0, cps, e_first, Nb, DECODE ? nullptr : perm, ring);
 
   if (DECODE && C > 1) cluster_wait();
 }
