@@ -231,15 +231,20 @@ class Prefill:
         return [t.empty(self.cache.unit_shape() + (self.N,), dtype=t.int32, device=self.device)
                 for _ in range(k)]
 
-    def step(self, kept=None, ev=None):
-        vd = self.vd
+    def append_next(self):
         k, v = self.blocks[self.i % len(self.blocks)]
         self.i += 1
-        vd.vd_append(self.cache, k, v, self.B)
+        self.vd.vd_append(self.cache, k, v, self.B)
+
+    def evict(self, kept=None, scores=None):
+        self.vd.vd_evict_block(self.cache, self.N, None, self.B, self.variant, self.mu,
+                               self.rs if self.mu else None, kept, scores)
+
+    def step(self, kept=None, ev=None):
+        self.append_next()
         if ev is not None:
             ev[0].record()
-        vd.vd_evict_block(self.cache, self.N, None, self.B, self.variant, self.mu,
-                          self.rs if self.mu else None, kept, None)
+        self.evict(kept)
         if ev is not None:
             ev[1].record()
 
@@ -341,15 +346,21 @@ class Decode:
         return [t.empty(self.cache.unit_shape(), dtype=t.int32, device=self.device)
                 for _ in range(k)]
 
-    def step(self, kept=None, ev=None):
-        vd = self.vd
-        k, v = self.tokens[self.i % len(self.tokens)]
+    def append_next(self, k=None, v=None):
+        if k is None:
+            k, v = self.tokens[self.i % len(self.tokens)]
         self.i += 1
-        vd.vd_append(self.cache, k, v, 1)
+        self.vd.vd_append(self.cache, k, v, 1)
+
+    def evict(self, evicted=None, kept=None, scores=None):
+        self.vd.vd_evict_decode(self.cache, self.N, None, self.variant, self.mu,
+                                self.rs if self.mu else None, evicted, kept, scores)
+
+    def step(self, kept=None, ev=None):
+        self.append_next()
         if ev is not None:
             ev[0].record()
-        vd.vd_evict_decode(self.cache, self.N, None, self.variant, self.mu,
-                           self.rs if self.mu else None, kept, None, None)
+        self.evict(kept)
         if ev is not None:
             ev[1].record()
 
