@@ -195,6 +195,9 @@ class Prefill:
     """Block boundary at steady state: append B rows, evict N + B -> N."""
 
     def __init__(self, name, cfg, device, seed, mu, variant, n_blocks=8):
+        """n_blocks distinct appended blocks are pre-generated and reused in
+        order; the benchmark asks for as many as the prompt has (T / B), so
+        every timed event appends rows the cache has not seen."""
         import torch
         import paper_2609_23314_gb300 as vd
         from paper_2609_23314_gb300 import workloads as wl
@@ -310,6 +313,8 @@ class Decode:
     """Decode step at steady state: append one token, evict N + 1 -> N."""
 
     def __init__(self, name, cfg, device, seed, mu, variant, n_tokens=8):
+        """n_tokens distinct appended tokens are pre-generated and reused in
+        order (the benchmark asks for the workload's 1024 decode steps)."""
         import torch
         import paper_2609_23314_gb300 as vd
         from paper_2609_23314_gb300 import workloads as wl
@@ -411,20 +416,26 @@ class Decode:
         return kk, vv, self.N + 1, self.N
 
 
-def make_workload(name, device, seed, mu, variant, n_seq=None):
+def make_workload(name, device, seed, mu, variant, n_seq=None, events=8):
+    """`events` = warm-up + timed steps: that many distinct blocks / tokens are
+    pre-generated, up to the workload's own length (T / B blocks of the
+    prompt, or its decode steps); longer runs reuse them in order."""
     from paper_2609_23314_gb300 import workloads as wl
     _, cfg = wl.config(name)
     if n_seq:
         cfg["n_seq"] = n_seq
     if cfg["kind"] == "prefill":
-        return Prefill(name, cfg, device, seed, mu, variant)
+        pool = max(8, min(events, cfg["T"] // cfg["B"]))
+        return Prefill(name, cfg, device, seed, mu, variant, n_blocks=pool)
     if cfg["kind"] == "decode":
-        return Decode(name, cfg, device, seed, mu, variant)
+        pool = max(8, min(events, cfg["steps"]))
+        return Decode(name, cfg, device, seed, mu, variant, n_tokens=pool)
     # ratio budget: its largest event is a decode step at N = 25% of the final length
     cfg = dict(cfg)
     total = cfg["prompt"] + cfg["gen_tokens"]
     cfg["N"] = wl.budget_at(cfg, total)
-    return Decode(name, cfg, device, seed, mu, variant)
+    pool = max(8, min(events, cfg["gen_tokens"]))
+    return Decode(name, cfg, device, seed, mu, variant, n_tokens=pool)
 
 
 # ---------------------------------------------------------------------------
@@ -529,7 +540,7 @@ def run_vd(args):
         if args.n_seq:
             cfg["n_seq"] = args.n_seq
         w = make_workload(name, device, rank_seed(wl.BASE_SEED + cfg["index"], rank), mu, variant,
-                          args.n_seq)
+                          args.n_seq, events=args.warmup + steps)
         m = measure_gpu(w, steps, args.warmup, device, min(steps, args.e2e_steps))
         step_ms = max_over_ranks(m["step_ms"], device) / steps
         kern_ms = max_over_ranks(m["kern_ms"], device)
@@ -563,7 +574,7 @@ def run_vd(args):
         base = cpu_baseline(primary["w"])
     secondary = None
     if args.secondary not in ("", "none") and args.secondary != args.workload:
-        secondary = one(args.secondary, max(3, args.steps // 20))
+        secondary = one(args.secondary, args.secondary_steps)
     if rank == 0:
         w = primary["w"]
         line = {
@@ -648,6 +659,7 @@ def main(argv=None):
     ap.add_argument("--workload", default="prefill_wide")
     ap.add_argument("--secondary", default="decode_batched",
                     help="a second workload measured into the same line ('' to skip)")
+    ap.add_argument("--secondary-steps", type=int, default=50)
     ap.add_argument("--mu", choices=["running", "recompute"], default="running")
     ap.add_argument("--variant", choices=["l2", "dir", "norm"], default="l2")
     ap.add_argument("--e2e-steps", type=int, default=50)
@@ -658,7 +670,8 @@ def main(argv=None):
     if args.warmup < 3:
         ap.error("--warmup must be at least 3")
     if args.steps is None:
-        args.steps = 5 if args.impl == "reference" else 1000
+        # prefill_wide: 200 evicting block events of its 240 (all distinct blocks)
+        args.steps = 5 if args.impl == "reference" else 200
     if args.impl == "reference":
         run_reference(args)
     else:

@@ -24,6 +24,12 @@ NVCC_FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-Xcompil
               "-I", INCLUDE, "-I", CSRC] + ARCH
 
 
+def _extra_defines():
+    """Extra -D flags for tuning sweeps (environment VD_NVCC_DEFINES, e.g.
+    "-DVD_RING_ITEMS=3"); empty by default."""
+    return [f for f in os.environ.get("VD_NVCC_DEFINES", "").split() if f.startswith("-D")]
+
+
 def _nvcc() -> str:
     cand = os.path.join(os.environ.get("CUDA_HOME", "/usr/local/cuda"), "bin", "nvcc")
     return cand if os.path.exists(cand) else "nvcc"
@@ -53,7 +59,7 @@ def build(force: bool = False, verbose: bool = False) -> str:
 
     def compile_one(src):
         obj = os.path.join(BUILD_DIR, os.path.basename(src)[:-3] + ".o")
-        cmd = [nvcc] + NVCC_FLAGS + ["-c", src, "-o", obj]
+        cmd = [nvcc] + NVCC_FLAGS + _extra_defines() + ["-c", src, "-o", obj]
         if verbose:
             print(" ".join(cmd), flush=True)
         subprocess.run(cmd, check=True)

@@ -139,6 +139,10 @@ vd_status device_state(DeviceState** out) {
     st.status = static_cast<unsigned*>(ptr);
     st.sms = p.multiProcessorCount;
     st.smem_optin = (int)p.sharedMemPerBlockOptin;
+    if (cudaFuncSetAttribute(reinterpret_cast<const void*>(&vd_rsum_init_kernel),
+                             cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             st.smem_optin) != cudaSuccess)
+      return VD_ERR_CUDA;
     for (int var = 0; var < 3; ++var)
       for (int dec = 0; dec < 2; ++dec) {
         const void* kern = evict_kernel((vd_variant)var, dec != 0);
@@ -199,18 +203,19 @@ bool cluster_allowed(int c, int d) {
   return c == 1 || (total_chunks % c == 0 && total_chunks / c >= 4);
 }
 
-// CTAs per unit.  Every candidate C in {1, 2, 4, 8, 16} that keeps row
-// segments of at least 64 bytes of [K | V] is scored by how well its CTAs
-// fill whole waves of the GPU (resident CTAs per SM from the occupancy
-// calculator at that C's shared-memory size); larger clusters pay a small
-// penalty for their per-unit synchronisation.  VD_CLUSTER_SIZE (1, 2, 4, 8
-// or 16) overrides the choice, for tuning.
+// CTAs per unit: the smallest C in {1, 2, 4, 8, 16} that keeps row segments
+// of at least 64 bytes of [K | V] and whose CTAs either form one nearly full
+// wave (>= 85% of the resident slots at that C's shared-memory size) or at
+// least two waves, so that no short tail wave runs alone; with none such,
+// the largest allowed C.  (Measured on GB300: a 1.1-wave launch loses ~15%,
+// while larger clusters than needed pay for extra synchronisation and
+// narrower row segments.)  VD_CLUSTER_SIZE (1, 2, 4, 8 or 16) overrides the
+// choice, for tuning.
 int choose_cluster(const void* kern, long long units, int d, int capacity, bool with_select,
                    const DeviceState& st, size_t* smem_out) {
   const char* env = std::getenv("VD_CLUSTER_SIZE");
   const int want = env ? std::atoi(env) : 0;
-  int best_c = 1;
-  double best_score = -1.0;
+  int chosen = 0, largest = 1;
   for (int c = 1; c <= 16; c *= 2) {
     if (want >= 1 && c != want) continue;
     if (want < 1 && !cluster_allowed(c, d)) continue;
@@ -223,17 +228,16 @@ int choose_cluster(const void* kern, long long units, int d, int capacity, bool 
       continue;
     }
     if (occ < 1 || !cluster_fits(kern, units, c, smem)) continue;
-    const double slots = (double)st.sms * occ;
-    const double waves = (double)(units * c) / slots;
-    const double eff = waves <= 1.0 ? waves : waves / std::ceil(waves);
-    const double score = eff - 0.02 * std::log2((double)c);
-    if (score > best_score) {
-      best_score = score;
-      best_c = c;
+    largest = c;
+    const double waves = (double)(units * c) / ((double)st.sms * occ);
+    if (want >= 1 || (waves >= 0.85 && waves <= 1.0) || waves >= 2.0) {
+      chosen = c;
+      break;
     }
   }
-  *smem_out = vd::smem_layout(capacity, best_c, with_select).total;
-  return best_c;
+  if (chosen == 0) chosen = largest;
+  *smem_out = vd::smem_layout(capacity, chosen, with_select).total;
+  return chosen;
 }
 
 vd_status launch(const void* kern, long long units, int c, size_t smem, const vd::EvictArgs& a,

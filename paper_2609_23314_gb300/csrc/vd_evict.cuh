@@ -50,9 +50,24 @@
 
 namespace vd {
 
-// cp.async ring: kRingStages stages of kRingItems 16-byte copies per thread.
-constexpr int kRingStages = 4;
-constexpr int kRingItems = 2;
+// cp.async ring: kRingStages stages of kRingItems 16-byte copies per thread
+// (overridable at build time for tuning sweeps).
+#ifndef VD_RING_STAGES
+#define VD_RING_STAGES 4
+#endif
+#ifndef VD_RING_ITEMS
+#define VD_RING_ITEMS 2
+#endif
+// Resident CTAs per SM the block and decode kernels are compiled for (caps
+// registers per thread at 65536 / (256 * n)).
+#ifndef VD_BLOCK_MIN_CTAS
+#define VD_BLOCK_MIN_CTAS 4
+#endif
+#ifndef VD_DECODE_MIN_CTAS
+#define VD_DECODE_MIN_CTAS 4
+#endif
+constexpr int kRingStages = VD_RING_STAGES;
+constexpr int kRingItems = VD_RING_ITEMS;
 constexpr int kRingBytes = kRingStages * kRingItems * kThreads * 16;
 
 struct EvictArgs {
@@ -84,6 +99,7 @@ struct Smem {
   float muhat[256];
   float acc_hi[256];  // this CTA's partial column sums (read by peer CTAs)
   float acc_lo[256];
+  double snew[256];       // running mode: sum of the appended rows, per column
   uint32_t hist[2][256];  // this CTA's radix histograms (read by peers)
   uint32_t ghist[256];
   int scan[kWarps];
@@ -406,7 +422,8 @@ __device__ __forceinline__ void compact_slice(uint16_t* kb, uint16_t* vb, int d,
 }
 
 template <int VAR, bool DECODE>
-__global__ void __launch_bounds__(kThreads, DECODE ? 4 : 3) evict_kernel(const EvictArgs a) {
+__global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLOCK_MIN_CTAS)
+    evict_kernel(const EvictArgs a) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   Smem& S = *reinterpret_cast<Smem*>(smem_raw);
   const int C = a.cluster;
@@ -501,7 +518,10 @@ __global__ void __launch_bounds__(kThreads, DECODE ? 4 : 3) evict_kernel(const E
         t = ff_add(t, p);
       }
       double sum = (double)t.hi + (double)t.lo;
-      if (run) sum += a.running_sum[(size_t)u * d + tid];
+      if (run) {
+        S.snew[tid] = sum;
+        sum += a.running_sum[(size_t)u * d + tid];
+      }
       S.mu[tid] = (float)(sum / (double)n);
     }
     __syncthreads();
@@ -632,8 +652,10 @@ __global__ void __launch_bounds__(kThreads, DECODE ? 4 : 3) evict_kernel(const E
   if (DECODE && a.evicted_out && rank == 0 && tid == 0) a.evicted_out[u] = e_first;
 
   // ---- 5. running sum: S += appended rows - evicted rows (own V columns) --
+  // The appended rows were already summed for the mean (all but Norm); only
+  // the evicted rows are read again.
   if (a.mu_running && vchunks > 0) {
-    const int B = a.B;
+    const int B = VAR != 2 ? 0 : a.B;
     sum_rows(vb, d, vchunk0, vchunks, vp, B + (n - Nb),
              [&](int i) {
                return i < B ? first_new + i : (DECODE ? e_first : (int)perm[Nb + (i - B)]);
@@ -642,7 +664,8 @@ __global__ void __launch_bounds__(kThreads, DECODE ? 4 : 3) evict_kernel(const E
     if (tid < vchunks * 8) {
       const int c = vchunk0 * 8 + tid;
       double* sp = a.running_sum + (size_t)u * d + c;
-      *sp = *sp + (double)S.acc_hi[c] + (double)S.acc_lo[c];
+      const double added = VAR != 2 ? S.snew[c] : 0.0;
+      *sp = *sp + added + (double)S.acc_hi[c] + (double)S.acc_lo[c];
     }
   }
 
