@@ -271,29 +271,34 @@ class Prefill:
         extra = self.U * d * 8 * 2 if self.mu else 0
         return v_read + move + extra, v_read + self.U * self.N * d * 2 * 2 * 2 + extra
 
-    # e2e through the C ABI with host buffers
-    def e2e_setup(self):
+    # e2e through the C ABI with host buffers (see run_e2e)
+    def e2e_setup(self, pool):
         t = self.torch
         us = self.cache.unit_shape()
-        self.h_blocks = [(k.cpu().pin_memory(), v.cpu().pin_memory()) for k, v in self.blocks[:2]]
-        self.d_k = t.empty(us + (self.B, self.d), dtype=t.bfloat16, device=self.device)
-        self.d_v = t.empty_like(self.d_k)
-        self.d_kept = t.empty(us + (self.N,), dtype=t.int32, device=self.device)
-        self.h_kept = t.empty(us + (self.N,), dtype=t.int32).pin_memory()
-        bi = 2 * self.d_k.numel() * 2
-        bo = self.d_kept.numel() * 4
-        return bi, bo
+        self.h_in = [(k.cpu().pin_memory(), v.cpu().pin_memory())
+                     for k, v in self.blocks[:max(1, min(pool, len(self.blocks)))]]
+        self.d_in = [(t.empty(us + (self.B, self.d), dtype=t.bfloat16, device=self.device),
+                      t.empty(us + (self.B, self.d), dtype=t.bfloat16, device=self.device))
+                     for _ in range(2)]
+        self.d_out = [t.empty(us + (self.N,), dtype=t.int32, device=self.device) for _ in range(2)]
+        self.h_out = [t.empty(us + (self.N,), dtype=t.int32).pin_memory() for _ in range(2)]
+        return 2 * self.d_in[0][0].numel() * 2, self.d_out[0].numel() * 4
 
-    def e2e_step(self):
+    def e2e_h2d(self, i, b):
+        hk, hv = self.h_in[i % len(self.h_in)]
+        self.d_in[b][0].copy_(hk, non_blocking=True)
+        self.d_in[b][1].copy_(hv, non_blocking=True)
+
+    def e2e_compute(self, b):
         vd = self.vd
-        hk, hv = self.h_blocks[self.i % 2]
-        self.i += 1
-        self.d_k.copy_(hk, non_blocking=True)
-        self.d_v.copy_(hv, non_blocking=True)
-        vd.vd_append(self.cache, self.d_k, self.d_v, self.B)
-        vd.vd_evict_block(self.cache, self.N, None, self.B, self.variant, self.mu,
-                          self.rs if self.mu else None, self.d_kept, None)
-        self.h_kept.copy_(self.d_kept, non_blocking=True)
+        vd.vd_append(self.cache, self.d_in[b][0], self.d_in[b][1], self.B)
+
+    def e2e_evict(self, b):
+        self.vd.vd_evict_block(self.cache, self.N, None, self.B, self.variant, self.mu,
+                               self.rs if self.mu else None, self.d_out[b], None)
+
+    def e2e_d2h(self, b):
+        self.h_out[b].copy_(self.d_out[b], non_blocking=True)
 
     # oracle sample: the pre-eviction bytes of a few units at steady state
     def oracle_sample(self, units):
@@ -382,26 +387,32 @@ class Decode:
         extra = self.U * d * 8 * 2 if self.mu else 0
         return v_read + move + extra, v_read + self.U * self.N * d * 2 * 2 * 2 + extra
 
-    def e2e_setup(self):
+    def e2e_setup(self, pool):
         t = self.torch
         us = self.cache.unit_shape()
-        self.h_tokens = [(k.cpu().pin_memory(), v.cpu().pin_memory()) for k, v in self.tokens[:2]]
-        self.d_k = t.empty(us + (1, self.d), dtype=t.bfloat16, device=self.device)
-        self.d_v = t.empty_like(self.d_k)
-        self.d_ev = t.empty(us, dtype=t.int32, device=self.device)
-        self.h_ev = t.empty(us, dtype=t.int32).pin_memory()
-        return 2 * self.d_k.numel() * 2, self.d_ev.numel() * 4
+        self.h_in = [(k.cpu().pin_memory(), v.cpu().pin_memory())
+                     for k, v in self.tokens[:max(1, min(pool, len(self.tokens)))]]
+        self.d_in = [(t.empty(us + (1, self.d), dtype=t.bfloat16, device=self.device),
+                      t.empty(us + (1, self.d), dtype=t.bfloat16, device=self.device))
+                     for _ in range(2)]
+        self.d_out = [t.empty(us, dtype=t.int32, device=self.device) for _ in range(2)]
+        self.h_out = [t.empty(us, dtype=t.int32).pin_memory() for _ in range(2)]
+        return 2 * self.d_in[0][0].numel() * 2, self.d_out[0].numel() * 4
 
-    def e2e_step(self):
-        vd = self.vd
-        hk, hv = self.h_tokens[self.i % 2]
-        self.i += 1
-        self.d_k.copy_(hk, non_blocking=True)
-        self.d_v.copy_(hv, non_blocking=True)
-        vd.vd_append(self.cache, self.d_k, self.d_v, 1)
-        vd.vd_evict_decode(self.cache, self.N, None, self.variant, self.mu,
-                           self.rs if self.mu else None, self.d_ev, None, None)
-        self.h_ev.copy_(self.d_ev, non_blocking=True)
+    def e2e_h2d(self, i, b):
+        hk, hv = self.h_in[i % len(self.h_in)]
+        self.d_in[b][0].copy_(hk, non_blocking=True)
+        self.d_in[b][1].copy_(hv, non_blocking=True)
+
+    def e2e_compute(self, b):
+        self.vd.vd_append(self.cache, self.d_in[b][0], self.d_in[b][1], 1)
+
+    def e2e_evict(self, b):
+        self.vd.vd_evict_decode(self.cache, self.N, None, self.variant, self.mu,
+                                self.rs if self.mu else None, self.d_out[b], None, None)
+
+    def e2e_d2h(self, b):
+        self.h_out[b].copy_(self.d_out[b], non_blocking=True)
 
     def oracle_sample(self, units):
         t = self.torch
@@ -441,6 +452,51 @@ def make_workload(name, device, seed, mu, variant, n_seq=None, events=8):
 # ---------------------------------------------------------------------------
 # measurement
 # ---------------------------------------------------------------------------
+def run_e2e(w, steps, device):
+    """Steps through the C ABI with the step's new rows copied in from pinned
+    host memory and its result (kept slots, or evicted slots for decode)
+    copied back, every step.  Three streams overlap the copies with the
+    eviction: copy-in (staging buffer b = step % 2), compute (append from the
+    staging buffer, then evict), copy-out; events keep a staging or result
+    buffer from being reused before its consumer is done.  Returns the time
+    from the first copy-in to the last copy-out (ms)."""
+    import torch
+    comp = torch.cuda.current_stream()
+    h2d, d2h = torch.cuda.Stream(), torch.cuda.Stream()
+    ev = lambda: torch.cuda.Event()
+    copied, free, done, out = [ev(), ev()], [ev(), ev()], [ev(), ev()], [ev(), ev()]
+    for b in range(2):
+        free[b].record(comp)
+        out[b].record(comp)
+    barrier(device)
+    torch.cuda.synchronize()
+    start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    start.record(comp)
+    h2d.wait_stream(comp)
+    d2h.wait_stream(comp)
+    for i in range(steps):
+        b = i % 2
+        with torch.cuda.stream(h2d):
+            h2d.wait_event(free[b])
+            w.e2e_h2d(i, b)
+            copied[b].record(h2d)
+        comp.wait_event(copied[b])
+        w.e2e_compute(b)
+        free[b].record(comp)
+        comp.wait_event(out[b])
+        w.e2e_evict(b)
+        done[b].record(comp)
+        with torch.cuda.stream(d2h):
+            d2h.wait_event(done[b])
+            w.e2e_d2h(b)
+            out[b].record(d2h)
+    comp.wait_stream(d2h)
+    comp.wait_stream(h2d)
+    stop.record(comp)
+    torch.cuda.synchronize()
+    return start.elapsed_time(stop)
+
+
 def measure_gpu(w, steps, warmup, device, e2e_steps):
     import torch
     for _ in range(warmup):
@@ -468,18 +524,9 @@ def measure_gpu(w, steps, warmup, device, e2e_steps):
     kern_ms = sum(a.elapsed_time(b) for a, b in evs) / steps
     moved = w.moved_rows(kept)
     # end to end through the C ABI with host buffers
-    bi, bo = w.e2e_setup()
-    for _ in range(min(3, warmup)):
-        w.e2e_step()
-    torch.cuda.synchronize()
-    barrier(device)
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    e0.record()
-    for _ in range(e2e_steps):
-        w.e2e_step()
-    e1.record()
-    torch.cuda.synchronize()
-    e2e_ms = e0.elapsed_time(e1)
+    bi, bo = w.e2e_setup(e2e_steps)
+    run_e2e(w, min(3, warmup), device)
+    e2e_ms = run_e2e(w, e2e_steps, device)
     status = w.vd.vd_get_device_status()
     if status != 0:
         raise RuntimeError(f"device status {status}: {w.vd.vd_status_string(status)}")
