@@ -135,6 +135,39 @@ vd_status vd_evict_decode(const vd_cache* c, int32_t N, const int32_t* N_dev, vd
                           vd_mu_mode mu, double* running_sum, int32_t* evicted_out,
                           int32_t* kept_idx_out, float* scores_out, vd_stream_t stream);
 
+/* Hole-fill layout (not in the paper; its eviction rule with a cache layout
+ * that moves as few rows as possible).  Same policy as vd_evict_block /
+ * vd_evict_decode (Sec. 2.1, Eq. eviction; Sec. 2.2, Eq. block_processing),
+ * but surviving rows are not kept in slot order: after the call, the kept
+ * rows that sat at or above the budget N_s (the appended ones) have moved
+ * into the evicted slots below N_s (paired in ascending order), every other
+ * kept row stays where it was, and slots [0, N_s) hold the surviving tokens
+ * in no particular order.  The tie-break is by token position instead of
+ * slot: among equal scores the lower position (earlier token) survives.
+ *   pos            int32 device [n_seq][n_layer][n_kv_head][capacity]: the
+ *                  sequence position of the token in each slot.  On entry,
+ *                  valid for rows [0, len - B); on exit, for rows [0, new len)
+ *                  (the kernel writes the positions of the appended rows and
+ *                  of every moved row).  Positions within a unit must be
+ *                  distinct and non-negative.
+ *   pos_first_new  int32 device [n_seq]: the position of the first appended
+ *                  row (slot len - B); appended row i has position
+ *                  pos_first_new[s] + i.
+ *   kept_idx_out   [..][N]: for every slot r < N_s, the pre-eviction slot of
+ *                  the token now in slot r (r itself unless r was refilled).
+ * A decode step therefore moves at most one row instead of shifting the cache
+ * tail; a block boundary moves at most B rows. */
+vd_status vd_evict_block_holefill(const vd_cache* c, int32_t N, const int32_t* N_dev, int32_t B,
+                                  vd_variant var, vd_mu_mode mu, double* running_sum,
+                                  int32_t* pos, const int32_t* pos_first_new,
+                                  int32_t* kept_idx_out, float* scores_out, vd_stream_t stream);
+
+vd_status vd_evict_decode_holefill(const vd_cache* c, int32_t N, const int32_t* N_dev,
+                                   vd_variant var, vd_mu_mode mu, double* running_sum,
+                                   int32_t* pos, const int32_t* pos_first_new,
+                                   int32_t* evicted_out, int32_t* kept_idx_out, float* scores_out,
+                                   vd_stream_t stream);
+
 /* Append B new rows per unit at slots [len, len + B) and set len += B (the
  * block append of Eq. block_processing).  k_new, v_new: bf16 device
  * [n_seq][n_layer][n_kv_head][B][head_dim], 16-B aligned.  A sequence with

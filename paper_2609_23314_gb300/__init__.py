@@ -20,7 +20,8 @@ import threading
 
 __all__ = [
     "VD_SCORE_L2", "VD_SCORE_DIR", "VD_SCORE_NORM", "VD_MU_RECOMPUTE", "VD_MU_RUNNING",
-    "VdError", "Cache", "vd_score", "vd_evict_block", "vd_evict_decode", "vd_append",
+    "VdError", "Cache", "vd_score", "vd_evict_block", "vd_evict_decode",
+    "vd_evict_block_holefill", "vd_evict_decode_holefill", "vd_append",
     "vd_running_sum_init", "vd_workspace_size", "vd_status_string", "vd_get_device_status",
     "library_path", "load_library",
 ]
@@ -66,6 +67,8 @@ def load_library() -> ctypes.CDLL:
             lib.vd_score.argtypes = [cp, S, P, P]
             lib.vd_evict_block.argtypes = [cp, I32, P, I32, S, S, P, P, P, P]
             lib.vd_evict_decode.argtypes = [cp, I32, P, S, S, P, P, P, P, P]
+            lib.vd_evict_block_holefill.argtypes = [cp, I32, P, I32, S, S, P, P, P, P, P, P]
+            lib.vd_evict_decode_holefill.argtypes = [cp, I32, P, S, S, P, P, P, P, P, P, P]
             lib.vd_append.argtypes = [cp, P, P, I32, P]
             lib.vd_running_sum_init.argtypes = [cp, P, P]
             lib.vd_workspace_size.argtypes = [cp]
@@ -73,8 +76,9 @@ def load_library() -> ctypes.CDLL:
             lib.vd_status_string.argtypes = [S]
             lib.vd_status_string.restype = ctypes.c_char_p
             lib.vd_get_device_status.argtypes = [P]
-            for f in ("vd_score", "vd_evict_block", "vd_evict_decode", "vd_append",
-                      "vd_running_sum_init", "vd_get_device_status"):
+            for f in ("vd_score", "vd_evict_block", "vd_evict_decode", "vd_evict_block_holefill",
+                      "vd_evict_decode_holefill", "vd_append", "vd_running_sum_init",
+                      "vd_get_device_status"):
                 getattr(lib, f).restype = S
             _lib = lib
         return _lib
@@ -195,6 +199,52 @@ def vd_evict_decode(cache: Cache, N: int, N_dev=None, variant: int = VD_SCORE_L2
     _check(load_library().vd_evict_decode(cache.ref(), int(N), args[0], int(variant), int(mu),
                                           args[1], args[2], args[3], args[4], _stream(stream)),
            "vd_evict_decode")
+
+
+def vd_evict_block_holefill(cache: Cache, N: int, pos, pos_first_new, N_dev=None, B: int = 0,
+                            variant: int = VD_SCORE_L2, mu: int = VD_MU_RECOMPUTE,
+                            running_sum=None, kept_idx_out=None, scores_out=None,
+                            stream=None) -> None:
+    """Block eviction in the hole-fill layout (kept appended rows move into the
+    evicted slots; ties by token position).  pos: int32 [.., capacity]
+    positions of the cached rows; pos_first_new: int32 [n_seq]."""
+    torch = _torch()
+    us = cache.unit_shape()
+    args = (
+        _ptr(N_dev, torch.int32, (cache.n_seq,), "N_dev", cache.device),
+        _ptr(running_sum, torch.float64, us + (cache.head_dim,), "running_sum", cache.device),
+        _ptr(pos, torch.int32, us + (cache.capacity,), "pos", cache.device),
+        _ptr(pos_first_new, torch.int32, (cache.n_seq,), "pos_first_new", cache.device),
+        _ptr(kept_idx_out, torch.int32, us + (int(N),), "kept_idx_out", cache.device),
+        _ptr(scores_out, torch.float32, us + (cache.capacity,), "scores_out", cache.device),
+    )
+    _check(load_library().vd_evict_block_holefill(cache.ref(), int(N), args[0], int(B), int(variant),
+                                                  int(mu), args[1], args[2], args[3], args[4],
+                                                  args[5], _stream(stream)),
+           "vd_evict_block_holefill")
+
+
+def vd_evict_decode_holefill(cache: Cache, N: int, pos, pos_first_new, N_dev=None,
+                             variant: int = VD_SCORE_L2, mu: int = VD_MU_RECOMPUTE,
+                             running_sum=None, evicted_out=None, kept_idx_out=None,
+                             scores_out=None, stream=None) -> None:
+    """Decode eviction in the hole-fill layout: the appended token moves into
+    the evicted slot (at most one row moves)."""
+    torch = _torch()
+    us = cache.unit_shape()
+    args = (
+        _ptr(N_dev, torch.int32, (cache.n_seq,), "N_dev", cache.device),
+        _ptr(running_sum, torch.float64, us + (cache.head_dim,), "running_sum", cache.device),
+        _ptr(pos, torch.int32, us + (cache.capacity,), "pos", cache.device),
+        _ptr(pos_first_new, torch.int32, (cache.n_seq,), "pos_first_new", cache.device),
+        _ptr(evicted_out, torch.int32, us, "evicted_out", cache.device),
+        _ptr(kept_idx_out, torch.int32, us + (int(N),), "kept_idx_out", cache.device),
+        _ptr(scores_out, torch.float32, us + (cache.capacity,), "scores_out", cache.device),
+    )
+    _check(load_library().vd_evict_decode_holefill(cache.ref(), int(N), args[0], int(variant),
+                                                   int(mu), args[1], args[2], args[3], args[4],
+                                                   args[5], args[6], _stream(stream)),
+           "vd_evict_decode_holefill")
 
 
 def vd_append(cache: Cache, k_new, v_new, B: int, stream=None) -> None:

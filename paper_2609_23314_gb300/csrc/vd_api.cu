@@ -264,7 +264,8 @@ vd_status launch(const void* kern, long long units, int c, size_t smem, const vd
 
 vd_status run(const vd_cache* c, int32_t N, const int32_t* N_dev, int32_t B, vd_variant var,
               vd_mu_mode mu, double* running_sum, int32_t* evicted_out, int32_t* kept_idx_out,
-              float* scores_out, cudaStream_t s, bool decode, bool score_only) {
+              float* scores_out, cudaStream_t s, bool decode, bool score_only,
+              int32_t* pos = nullptr, const int32_t* pos_new = nullptr) {
   vd_status r = validate_cache(c);
   if (r != VD_OK) return r;
   if (var != VD_SCORE_L2 && var != VD_SCORE_DIR && var != VD_SCORE_NORM) return VD_ERR_INVALID_ARG;
@@ -276,6 +277,8 @@ vd_status run(const vd_cache* c, int32_t N, const int32_t* N_dev, int32_t B, vd_
   } else if (!scores_out) {
     return VD_ERR_INVALID_ARG;
   }
+  const bool holefill = pos != nullptr || pos_new != nullptr;
+  if (holefill && (!pos || !pos_new)) return VD_ERR_INVALID_ARG;
   DeviceState* st = nullptr;
   r = device_state(&st);
   if (r != VD_OK) return r;
@@ -306,6 +309,9 @@ vd_status run(const vd_cache* c, int32_t N, const int32_t* N_dev, int32_t B, vd_
   a.B = decode ? 1 : B;
   a.mu_running = (!score_only && mu == VD_MU_RUNNING) ? 1 : 0;
   a.score_only = score_only ? 1 : 0;
+  a.pos = pos;
+  a.pos_new = pos_new;
+  a.holefill = holefill ? 1 : 0;
   size_t smem = 0;
   a.cluster = choose_cluster(kern, units, c->head_dim, c->capacity, !small, *st, &smem);
   if (smem > (size_t)st->smem_optin) return VD_ERR_UNSUPPORTED;
@@ -343,6 +349,25 @@ vd_status vd_evict_decode(const vd_cache* c, int32_t N, const int32_t* N_dev, vd
                           int32_t* kept_idx_out, float* scores_out, vd_stream_t stream) {
   return run(c, N, N_dev, 1, var, mu, running_sum, evicted_out, kept_idx_out, scores_out,
              reinterpret_cast<cudaStream_t>(stream), true, false);
+}
+
+vd_status vd_evict_block_holefill(const vd_cache* c, int32_t N, const int32_t* N_dev, int32_t B,
+                                  vd_variant var, vd_mu_mode mu, double* running_sum,
+                                  int32_t* pos, const int32_t* pos_first_new,
+                                  int32_t* kept_idx_out, float* scores_out, vd_stream_t stream) {
+  if (!pos || !pos_first_new) return VD_ERR_INVALID_ARG;
+  return run(c, N, N_dev, B, var, mu, running_sum, nullptr, kept_idx_out, scores_out,
+             reinterpret_cast<cudaStream_t>(stream), false, false, pos, pos_first_new);
+}
+
+vd_status vd_evict_decode_holefill(const vd_cache* c, int32_t N, const int32_t* N_dev,
+                                   vd_variant var, vd_mu_mode mu, double* running_sum,
+                                   int32_t* pos, const int32_t* pos_first_new,
+                                   int32_t* evicted_out, int32_t* kept_idx_out, float* scores_out,
+                                   vd_stream_t stream) {
+  if (!pos || !pos_first_new) return VD_ERR_INVALID_ARG;
+  return run(c, N, N_dev, 1, var, mu, running_sum, evicted_out, kept_idx_out, scores_out,
+             reinterpret_cast<cudaStream_t>(stream), true, false, pos, pos_first_new);
 }
 
 vd_status vd_append(const vd_cache* c, const void* k_new, const void* v_new, int32_t B,

@@ -89,6 +89,9 @@ struct EvictArgs {
   int32_t mu_running;     // 1: mean from running_sum + appended rows
   int32_t score_only;     // 1: vd_score (mean recomputed, no eviction)
   int32_t cluster;        // C, CTAs per unit
+  int32_t* pos;            // hole-fill layout: token positions [U][capacity]
+  const int32_t* pos_new;  // hole-fill layout: position of row len - B, [n_seq]
+  int32_t holefill;        // 1: hole-fill layout (ties by position), 0: ordered
 };
 
 // Fixed part of the dynamic shared memory.  After it (16-byte aligned): the
@@ -104,8 +107,11 @@ struct Smem {
   uint32_t ghist[256];
   int scan[kWarps];
   float fsh[kWarps];
-  unsigned long long best;  // decode: this CTA's (key, -slot) minimum
+  unsigned long long best;  // decode: this CTA's (key, -tie-break) minimum
   unsigned long long wbest[kWarps];
+  int best_slot;            // decode: the slot of `best`
+  int wslot[kWarps];
+  int holes;                // hole-fill: evicted slots below N
   int sel_digit, sel_above, sel_cnt;
   int cnt_gt, cnt_eq;  // this CTA's keys > t and == t (read by peers)
   int mu_zero;
@@ -241,15 +247,17 @@ __device__ __forceinline__ uint32_t score_key(float s, bool& bad) {
 
 // Radix select over the keys of the whole cluster: t = the N-th largest key
 // (1-based), keep_eq = how many keys equal to t survive, cnt_eq = how many
-// keys equal t.  `keys` holds this CTA's R keys.
+// keys equal t.  key_of(j, ok) gives the key of this CTA's j-th row (j < R)
+// and whether the row takes part.
 struct Selection {
   uint32_t t;
   int keep_eq;
   int cnt_eq;
 };
 
-__device__ __forceinline__ Selection cluster_radix_select(const uint32_t* keys, int R, int N,
-                                                          int C, Smem& S) {
+template <class KeyOf>
+__device__ __forceinline__ Selection cluster_radix_select(KeyOf key_of, int R, int N, int C,
+                                                          Smem& S) {
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   uint32_t prefix = 0, pmask = 0;
   int need = N, cnt = 0;
@@ -260,8 +268,10 @@ __device__ __forceinline__ Selection cluster_radix_select(const uint32_t* keys, 
     __syncthreads();
     for (int base = 0; base < R; base += kThreads) {
       const int j = base + tid;
-      const uint32_t key = j < R ? keys[j] : 0u;
-      const bool match = j < R && (key & pmask) == prefix;
+      bool ok = false;
+      uint32_t key = 0u;
+      if (j < R) key = key_of(j, ok);
+      const bool match = ok && (key & pmask) == prefix;
       const unsigned act = __ballot_sync(kFull, match);
       if (match) {
         const uint32_t dig = (key >> shift) & 255u;
@@ -324,17 +334,21 @@ __device__ __forceinline__ Selection cluster_radix_select(const uint32_t* keys, 
 // evicted slots ascending at [N, n).  Threads own contiguous row chunks, so
 // prefix sums follow slot order (ties go to the lower slot).  Ends with the
 // cluster barrier after which every CTA's perm[] is complete.
+template <class TieKey>
 __device__ __forceinline__ void cluster_build_perm(const uint32_t* keys, int r0, int R, int N,
-                                                   Selection sel, int C, unsigned rank,
+                                                   Selection sel, bool by_tiekey, uint32_t t2,
+                                                   TieKey tiekey, int C, unsigned rank,
                                                    uint16_t* perm, Smem& S) {
   const int tid = threadIdx.x;
   const int ch = (R + kThreads - 1) / kThreads;
   const int c0 = min(R, tid * ch), c1 = min(R, c0 + ch);
   const uint32_t t = sel.t;
+  // ordered layout: ties go to the lowest slots (prefix counts below);
+  // hole-fill layout: a tied row survives iff tiekey(j) >= t2
   int ngt = 0, neq = 0;
   for (int j = c0; j < c1; ++j) {
     ngt += keys[j] > t;
-    neq += keys[j] == t;
+    if (keys[j] == t) neq += by_tiekey ? (tiekey(j) >= t2) : 1;
   }
   int tot_gt, tot_eq;
   const int gt_ex = block_exclusive_scan(ngt, S.scan, tot_gt);
@@ -350,17 +364,18 @@ __device__ __forceinline__ void cluster_build_perm(const uint32_t* keys, int r0,
   for (int rr = 0; rr < (int)rank; ++rr) {
     const int g = (int)ld_cluster_u32(mapa(smem_addr(&S.cnt_gt), rr));
     const int e = (int)ld_cluster_u32(mapa(smem_addr(&S.cnt_eq), rr));
-    kept_off += g + min(max(q - tie_off, 0), e);
+    kept_off += g + (by_tiekey ? e : min(max(q - tie_off, 0), e));
     tie_off += e;
   }
   const int my_tie_quota = max(q - tie_off, 0);  // ties this CTA may still keep
   int tie_rank = eq_ex;                          // ties of this CTA before the chunk
-  int kp = kept_off + gt_ex + min(my_tie_quota, eq_ex);
+  int kp = kept_off + gt_ex + (by_tiekey ? eq_ex : min(my_tie_quota, eq_ex));
   const uint32_t perm_addr = smem_addr(perm);
   for (int j = c0; j < c1; ++j) {
     const uint32_t key = keys[j];
     const bool eq = key == t;
-    const bool keep = key > t || (eq && tie_rank < my_tie_quota);
+    const bool keep =
+        key > t || (eq && (by_tiekey ? tiekey(j) >= t2 : tie_rank < my_tie_quota));
     tie_rank += eq;
     const int row = r0 + j;
     const int pos = keep ? kp : N + (row - kp);
@@ -421,6 +436,35 @@ __device__ __forceinline__ void compact_slice(uint16_t* kb, uint16_t* vb, int d,
   cp_async_wait<0>();
 }
 
+// Hole-fill layout: move h rows, row src_of(i) -> row dst_of(i), of the
+// column slice [chunk0, chunk0 + cps) of [K | V].  Every source lies at or
+// above N and every destination below it, so the moves are independent.
+template <class SrcOf, class DstOf>
+__device__ __forceinline__ void move_rows(uint16_t* kb, uint16_t* vb, int d, int chunk0, int cps,
+                                          int h, SrcOf src_of, DstOf dst_of) {
+  const int d8 = d >> 3;
+  const int items = h * cps;
+  constexpr int U = 4;
+  for (int base = threadIdx.x; base < items; base += kThreads * U) {
+    uint4 q[U];
+    uint16_t* dstp[U];
+#pragma unroll
+    for (int k = 0; k < U; ++k) {
+      const int it = base + k * kThreads;
+      dstp[k] = nullptr;
+      if (it < items) {
+        const int i = it / cps, c = chunk0 + it % cps;
+        uint16_t* col = c < d8 ? kb + c * 8 : vb + (c - d8) * 8;
+        q[k] = ld_cg16(col + (size_t)src_of(i) * d);
+        dstp[k] = col + (size_t)dst_of(i) * d;
+      }
+    }
+#pragma unroll
+    for (int k = 0; k < U; ++k)
+      if (dstp[k]) st16(dstp[k], q[k]);
+  }
+}
+
 template <int VAR, bool DECODE>
 __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLOCK_MIN_CTAS)
     evict_kernel(const EvictArgs a) {
@@ -468,8 +512,16 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
   int vp = 1;
   while (vp < vchunks) vp <<= 1;
   const int first_new = n - a.B;
+  // hole-fill layout: token positions (rows at or above first_new are the
+  // appended ones, numbered from pos_new)
+  const bool hf = a.holefill != 0 && !a.score_only;
+  int32_t* posu = hf ? a.pos + (size_t)u * a.capacity : nullptr;
+  const int pnew = hf ? a.pos_new[seq] : 0;
+  auto pos_of = [&](int r) -> int { return r < first_new ? posu[r] : pnew + (r - first_new); };
 
   if (!evict && !a.score_only) {
+    if (hf && rank == 0)
+      for (int r = max(first_new, 0) + tid; r < n; r += kThreads) posu[r] = pnew + (r - first_new);
     // ---- nothing to evict: identity outputs, running sum += appended rows ---
     if (a.kept_out)
       for (int i = (int)rank * kThreads + tid; i < a.N; i += C * kThreads)
@@ -550,6 +602,7 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
     }
     const bool mu_zero = VAR == 1 && S.mu_zero;
     unsigned long long best = ~0ull;
+    int best_slot = 0;
     float* sc_out = a.scores_out ? a.scores_out + (size_t)u * a.capacity : nullptr;
     stream_rows(
         vb, d, 0, d8, lpr, r1 - r0, [&](int i) { return r0 + i; },
@@ -595,9 +648,15 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
               const uint32_t key = score_key(s, bad);
               if (bad) record_status(a.status, kStNonfinite);
               if (DECODE) {
-                const unsigned long long pk = ((unsigned long long)key << 32) |
-                                              (unsigned long long)(0xffffffffu - (unsigned)r);
-                best = pk < best ? pk : best;
+                // lowest score first; among equal scores the latest token
+                // (highest slot, or highest position in the hole-fill layout)
+                const unsigned tb = hf ? (unsigned)pos_of(r) : (unsigned)r;
+                const unsigned long long pk =
+                    ((unsigned long long)key << 32) | (unsigned long long)(0xffffffffu - tb);
+                if (pk < best) {
+                  best = pk;
+                  best_slot = r;
+                }
               } else {
                 keys[item] = key;
               }
@@ -610,13 +669,30 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
       return;
     }
     if (DECODE) {
-      best = warp_min_u64(best);
-      if (lane == 0) S.wbest[warp] = best;
+#pragma unroll
+      for (int off = 16; off > 0; off >>= 1) {
+        const unsigned long long o = __shfl_xor_sync(kFull, best, off);
+        const int os = __shfl_xor_sync(kFull, best_slot, off);
+        if (o < best) {
+          best = o;
+          best_slot = os;
+        }
+      }
+      if (lane == 0) {
+        S.wbest[warp] = best;
+        S.wslot[warp] = best_slot;
+      }
       __syncthreads();
       if (tid == 0) {
         unsigned long long b = ~0ull;
-        for (int w = 0; w < kWarps; ++w) b = S.wbest[w] < b ? S.wbest[w] : b;
+        int bs = 0;
+        for (int w = 0; w < kWarps; ++w)
+          if (S.wbest[w] < b) {
+            b = S.wbest[w];
+            bs = S.wslot[w];
+          }
         S.best = b;
+        S.best_slot = bs;
       }
     }
   }
@@ -626,22 +702,46 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
   if (DECODE) {
     if (C > 1) cluster_sync(); else __syncthreads();
     unsigned long long b = ~0ull;
+    int bs = 0;
     for (int rr = 0; rr < C; ++rr) {
       const unsigned long long o =
           C > 1 ? ld_cluster_u64(mapa(smem_addr(&S.best), rr)) : S.best;
-      b = o < b ? o : b;
+      const int os = C > 1 ? (int)ld_cluster_u32(mapa(smem_addr(&S.best_slot), rr)) : S.best_slot;
+      if (o < b) {
+        b = o;
+        bs = os;
+      }
     }
     if (C > 1) cluster_arrive();  // last peer access of this CTA; wait before exit
-    e_first = (int)(0xffffffffu - (unsigned)(b & 0xffffffffull));
+    e_first = bs;
   } else {
     __syncthreads();  // own keys complete
-    const Selection sel = cluster_radix_select(keys, r1 - r0, Nb, C, S);
-    cluster_build_perm(keys, r0, r1 - r0, Nb, sel, C, rank, perm, S);
+    const int R = r1 - r0;
+    const Selection sel = cluster_radix_select(
+        [&](int j, bool& ok) {
+          ok = true;
+          return keys[j];
+        },
+        R, Nb, C, S);
+    // hole-fill layout: the surviving ties are the lowest positions, found
+    // by a second select over the complemented positions of the tied rows
+    uint32_t t2 = 0u;
+    if (hf && sel.cnt_eq > sel.keep_eq) {
+      const Selection s2 = cluster_radix_select(
+          [&](int j, bool& ok) {
+            ok = keys[j] == sel.t;
+            return ~(uint32_t)pos_of(r0 + j);
+          },
+          R, sel.keep_eq, C, S);
+      t2 = s2.t;
+    }
+    cluster_build_perm(keys, r0, R, Nb, sel, hf, t2,
+                       [&](int j) { return ~(uint32_t)pos_of(r0 + j); }, C, rank, perm, S);
     e_first = perm[Nb];
   }
 
   // ---- outputs -----------------------------------------------------------
-  if (a.kept_out) {
+  if (a.kept_out && !hf) {
     int32_t* ko = a.kept_out + (size_t)u * a.N;
     for (int i = (int)rank * kThreads + tid; i < a.N; i += C * kThreads) {
       int val = -1;
@@ -670,7 +770,43 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
   }
 
   // ---- 6. in-place compaction of this CTA's column slice ---------------
-  compact_slice(kb, vb, d, chunk0, cps, e_first, Nb, DECODE ? nullptr : perm, ring);
+  if (!hf) {
+    compact_slice(kb, vb, d, chunk0, cps, e_first, Nb, DECODE ? nullptr : perm, ring);
+  } else {
+    // hole-fill: the kept rows at or above N move into the evicted slots
+    // below N, in ascending order (movers: the tail of the kept list; holes:
+    // the head of the evicted list)
+    int h;
+    if (DECODE) {
+      h = e_first < Nb ? 1 : 0;
+    } else {
+      if (tid == 0) {
+        int lo = 0, hi = n - Nb;
+        while (lo < hi) {
+          const int mid = (lo + hi) >> 1;
+          if ((int)perm[Nb + mid] < Nb) lo = mid + 1; else hi = mid;
+        }
+        S.holes = lo;
+      }
+      __syncthreads();
+      h = S.holes;
+    }
+    auto src = [&](int i) { return DECODE ? n - 1 : (int)perm[Nb - h + i]; };
+    auto dst = [&](int i) { return DECODE ? e_first : (int)perm[Nb + i]; };
+    move_rows(kb, vb, d, chunk0, cps, h, src, dst);
+    if (rank == 0) {
+      for (int r = max(first_new, 0) + tid; r < Nb; r += kThreads) posu[r] = pnew + (r - first_new);
+      int32_t* ko = a.kept_out ? a.kept_out + (size_t)u * a.N : nullptr;
+      if (ko)
+        for (int r = tid; r < a.N; r += kThreads) ko[r] = r < Nb ? r : -1;
+      __syncthreads();
+      for (int i = tid; i < h; i += kThreads) {
+        const int sr = src(i), dr = dst(i);
+        posu[dr] = pos_of(sr);
+        if (ko) ko[dr] = sr;
+      }
+    }
+  }
 
   if (DECODE && C > 1) cluster_wait();
 }
