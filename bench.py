@@ -79,6 +79,31 @@ def barrier(device=None):
             dist.barrier()
 
 
+def bind_to_gpu_numa(gpu_index: int):
+    """Pins this process to the host CPUs local to the GPU (sysfs local_cpulist
+    of its PCI device), so pinned host buffers are allocated on the GPU's own
+    NUMA node; returns the CPU list or None."""
+    try:
+        bus = subprocess.run(["nvidia-smi", "-i", str(gpu_index), "--query-gpu=pci.bus_id",
+                              "--format=csv,noheader"], capture_output=True, text=True,
+                             timeout=20).stdout.strip()
+        dom, rest = bus.split(":", 1)
+        dev = f"{int(dom, 16):04x}:{rest}".lower()
+        with open(f"/sys/bus/pci/devices/{dev}/local_cpulist") as f:
+            spec = f.read().strip()
+        cpus = set()
+        for part in spec.split(","):
+            a, _, b = part.partition("-")
+            cpus.update(range(int(a), int(b or a) + 1))
+        cpus &= os.sched_getaffinity(0)
+        if cpus:
+            os.sched_setaffinity(0, cpus)
+            return spec
+    except Exception:
+        pass
+    return None
+
+
 def whole_job_rate(units_per_rank_step: float, steps: int, world: int, max_ms: float) -> float:
     return units_per_rank_step * steps * world / (max_ms / 1e3)
 
@@ -194,10 +219,11 @@ class ClockSampler:
 class Prefill:
     """Block boundary at steady state: append B rows, evict N + B -> N."""
 
-    def __init__(self, name, cfg, device, seed, mu, variant, n_blocks=8):
+    def __init__(self, name, cfg, device, seed, mu, variant, n_blocks=8, layout="ordered"):
         """n_blocks distinct appended blocks are pre-generated and reused in
         order; the benchmark asks for as many as the prompt has (T / B), so
-        every timed event appends rows the cache has not seen."""
+        every timed event appends rows the cache has not seen.  layout
+        "holefill" uses vd_evict_block_holefill with a token-position array."""
         import torch
         import paper_2609_23314_gb300 as vd
         from paper_2609_23314_gb300 import workloads as wl
@@ -225,6 +251,13 @@ class Prefill:
         self.kept = None
         self.i = 0
         self.launches_per_step = 4     # append + len add, evict + len clamp
+        self.holefill = layout == "holefill"
+        if self.holefill:
+            self.pos = torch.arange(self.cap, dtype=torch.int32, device=device).repeat(
+                self.U).view(us + (self.cap,)).contiguous()
+            steps = torch.arange(1 << 14, dtype=torch.int32, device=device)
+            self.pos_new_all = (self.N + self.B * steps).view(-1, 1).repeat(
+                1, cfg["n_seq"]).contiguous()
 
     def head_tokens_per_step(self):
         return self.U * (self.N + self.B)
@@ -240,8 +273,14 @@ class Prefill:
         self.vd.vd_append(self.cache, k, v, self.B)
 
     def evict(self, kept=None, scores=None):
-        self.vd.vd_evict_block(self.cache, self.N, None, self.B, self.variant, self.mu,
-                               self.rs if self.mu else None, kept, scores)
+        if self.holefill:
+            pn = self.pos_new_all[(self.i - 1) % self.pos_new_all.shape[0]]
+            self.vd.vd_evict_block_holefill(self.cache, self.N, self.pos, pn, None, self.B,
+                                            self.variant, self.mu, self.rs if self.mu else None,
+                                            kept, scores)
+        else:
+            self.vd.vd_evict_block(self.cache, self.N, None, self.B, self.variant, self.mu,
+                                   self.rs if self.mu else None, kept, scores)
 
     def step(self, kept=None, ev=None):
         self.append_next()
@@ -252,23 +291,33 @@ class Prefill:
             ev[1].record()
 
     def moved_rows(self, kept_list):
-        """Rows of one unit moved by the compaction: N - first evicted slot."""
+        """Rows moved per launch, all units: ordered layout, N - first evicted
+        slot per unit; hole-fill layout, the refilled slots (kept[r] != r)."""
         t = self.torch
         total = 0
         ar = t.arange(self.N, device=self.device, dtype=t.int32)
         for kp in kept_list:
             kk = kp.view(self.U, self.N)
             same = (kk == ar)
+            if self.holefill:
+                total += int((~same).sum().item())
+                continue
             first = t.where(same.all(dim=1), t.full((self.U,), self.N, device=self.device),
                             (~same).int().argmax(dim=1))
             total += int((self.N - first).sum().item())
         return total / max(1, len(kept_list))
 
     def bytes_per_launch(self, moved_rows_total):
+        """(algorithmic, nominal) bytes per launch: V read once, moved K and V
+        rows read and written, running-sum state (and, hole-fill, the moved
+        rows' positions)."""
         n, d = self.N + self.B, self.d
         v_read = self.U * n * d * 2
         move = moved_rows_total * d * 2 * 2 * 2
         extra = self.U * d * 8 * 2 if self.mu else 0
+        if self.holefill:
+            extra += moved_rows_total * 4 + self.U * self.B * 4
+            return v_read + move + extra, v_read + self.U * self.B * d * 2 * 2 * 2 + extra
         return v_read + move + extra, v_read + self.U * self.N * d * 2 * 2 * 2 + extra
 
     # e2e through the C ABI with host buffers (see run_e2e)
@@ -290,12 +339,11 @@ class Prefill:
         self.d_in[b][1].copy_(hv, non_blocking=True)
 
     def e2e_compute(self, b):
-        vd = self.vd
-        vd.vd_append(self.cache, self.d_in[b][0], self.d_in[b][1], self.B)
+        self.i += 1
+        self.vd.vd_append(self.cache, self.d_in[b][0], self.d_in[b][1], self.B)
 
     def e2e_evict(self, b):
-        self.vd.vd_evict_block(self.cache, self.N, None, self.B, self.variant, self.mu,
-                               self.rs if self.mu else None, self.d_out[b], None)
+        self.evict(self.d_out[b])
 
     def e2e_d2h(self, b):
         self.h_out[b].copy_(self.d_out[b], non_blocking=True)
@@ -317,9 +365,10 @@ class Prefill:
 class Decode:
     """Decode step at steady state: append one token, evict N + 1 -> N."""
 
-    def __init__(self, name, cfg, device, seed, mu, variant, n_tokens=8):
+    def __init__(self, name, cfg, device, seed, mu, variant, n_tokens=8, layout="ordered"):
         """n_tokens distinct appended tokens are pre-generated and reused in
-        order (the benchmark asks for the workload's 1024 decode steps)."""
+        order (the benchmark asks for the workload's 1024 decode steps).
+        layout "holefill" uses vd_evict_decode_holefill."""
         import torch
         import paper_2609_23314_gb300 as vd
         from paper_2609_23314_gb300 import workloads as wl
@@ -347,6 +396,12 @@ class Decode:
             vd.vd_running_sum_init(self.cache, self.rs)
         self.i = 0
         self.launches_per_step = 4
+        self.holefill = layout == "holefill"
+        if self.holefill:
+            self.pos = torch.arange(self.cap, dtype=torch.int32, device=device).repeat(
+                self.U).view(us + (self.cap,)).contiguous()
+            steps = torch.arange(1 << 14, dtype=torch.int32, device=device)
+            self.pos_new_all = (self.N + steps).view(-1, 1).repeat(1, cfg["n_seq"]).contiguous()
 
     def head_tokens_per_step(self):
         return self.U * (self.N + 1)
@@ -363,8 +418,14 @@ class Decode:
         self.vd.vd_append(self.cache, k, v, 1)
 
     def evict(self, evicted=None, kept=None, scores=None):
-        self.vd.vd_evict_decode(self.cache, self.N, None, self.variant, self.mu,
-                                self.rs if self.mu else None, evicted, kept, scores)
+        if self.holefill:
+            pn = self.pos_new_all[(self.i - 1) % self.pos_new_all.shape[0]]
+            self.vd.vd_evict_decode_holefill(self.cache, self.N, self.pos, pn, None, self.variant,
+                                             self.mu, self.rs if self.mu else None, evicted,
+                                             kept, scores)
+        else:
+            self.vd.vd_evict_decode(self.cache, self.N, None, self.variant, self.mu,
+                                    self.rs if self.mu else None, evicted, kept, scores)
 
     def step(self, kept=None, ev=None):
         self.append_next()
@@ -375,16 +436,28 @@ class Decode:
             ev[1].record()
 
     def moved_rows(self, evicted_list):
+        """Rows moved per launch, all units: ordered layout, N - evicted slot
+        per unit; hole-fill layout, one row per unit whose evicted slot lies
+        below N."""
         total = 0
         for e in evicted_list:
-            total += int((self.N - e.long()).sum().item())
+            if self.holefill:
+                total += int((e < self.N).sum().item())
+            else:
+                total += int((self.N - e.long()).sum().item())
         return total / max(1, len(evicted_list))
 
     def bytes_per_launch(self, moved_rows_total):
+        """(algorithmic, nominal) bytes per launch; hole-fill adds the
+        positions read for the tie-break (4 B per cached row) and written for
+        moved rows."""
         n, d = self.N + 1, self.d
         v_read = self.U * n * d * 2
         move = moved_rows_total * d * 2 * 2 * 2
         extra = self.U * d * 8 * 2 if self.mu else 0
+        if self.holefill:
+            extra += self.U * self.N * 4 + moved_rows_total * 4
+            return v_read + move + extra, v_read + self.U * d * 2 * 2 * 2 + extra
         return v_read + move + extra, v_read + self.U * self.N * d * 2 * 2 * 2 + extra
 
     def e2e_setup(self, pool):
@@ -405,11 +478,11 @@ class Decode:
         self.d_in[b][1].copy_(hv, non_blocking=True)
 
     def e2e_compute(self, b):
+        self.i += 1
         self.vd.vd_append(self.cache, self.d_in[b][0], self.d_in[b][1], 1)
 
     def e2e_evict(self, b):
-        self.vd.vd_evict_decode(self.cache, self.N, None, self.variant, self.mu,
-                                self.rs if self.mu else None, self.d_out[b], None, None)
+        self.evict(self.d_out[b])
 
     def e2e_d2h(self, b):
         self.h_out[b].copy_(self.d_out[b], non_blocking=True)
@@ -427,7 +500,7 @@ class Decode:
         return kk, vv, self.N + 1, self.N
 
 
-def make_workload(name, device, seed, mu, variant, n_seq=None, events=8):
+def make_workload(name, device, seed, mu, variant, n_seq=None, events=8, layout="ordered"):
     """`events` = warm-up + timed steps: that many distinct blocks / tokens are
     pre-generated, up to the workload's own length (T / B blocks of the
     prompt, or its decode steps); longer runs reuse them in order."""
@@ -437,16 +510,16 @@ def make_workload(name, device, seed, mu, variant, n_seq=None, events=8):
         cfg["n_seq"] = n_seq
     if cfg["kind"] == "prefill":
         pool = max(8, min(events, cfg["T"] // cfg["B"]))
-        return Prefill(name, cfg, device, seed, mu, variant, n_blocks=pool)
+        return Prefill(name, cfg, device, seed, mu, variant, n_blocks=pool, layout=layout)
     if cfg["kind"] == "decode":
         pool = max(8, min(events, cfg["steps"]))
-        return Decode(name, cfg, device, seed, mu, variant, n_tokens=pool)
+        return Decode(name, cfg, device, seed, mu, variant, n_tokens=pool, layout=layout)
     # ratio budget: its largest event is a decode step at N = 25% of the final length
     cfg = dict(cfg)
     total = cfg["prompt"] + cfg["gen_tokens"]
     cfg["N"] = wl.budget_at(cfg, total)
     pool = max(8, min(events, cfg["gen_tokens"]))
-    return Decode(name, cfg, device, seed, mu, variant, n_tokens=pool)
+    return Decode(name, cfg, device, seed, mu, variant, n_tokens=pool, layout=layout)
 
 
 # ---------------------------------------------------------------------------
@@ -573,6 +646,7 @@ def run_vd(args):
     else:
         torch.cuda.set_device(0)
     device = torch.device("cuda", torch.cuda.current_device())
+    host_cpus = bind_to_gpu_numa(device.index)
     if rank == 0:
         vd_build.build()
     barrier(device)
@@ -582,12 +656,12 @@ def run_vd(args):
     peak, peak_src = hbm_peak()
     from paper_2609_23314_gb300 import workloads as wl
 
-    def one(name, steps):
+    def one(name, steps, layout="ordered"):
         _, cfg = wl.config(name)
         if args.n_seq:
             cfg["n_seq"] = args.n_seq
         w = make_workload(name, device, rank_seed(wl.BASE_SEED + cfg["index"], rank), mu, variant,
-                          args.n_seq, events=args.warmup + steps)
+                          args.n_seq, events=args.warmup + steps, layout=layout)
         m = measure_gpu(w, steps, args.warmup, device, min(steps, args.e2e_steps))
         step_ms = max_over_ranks(m["step_ms"], device) / steps
         kern_ms = max_over_ranks(m["kern_ms"], device)
@@ -602,28 +676,45 @@ def run_vd(args):
                     "h2d_bytes_per_step": m["bi"], "d2h_bytes_per_step": m["bo"]},
             "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                          "frac": achieved / peak, "traffic": ncu_traffic(name),
-                         "kernel": f"vd::evict_kernel<{variant}, {'true' if isinstance(w, Decode) else 'false'}>",
+                         "kernel": f"vd::evict_kernel<{variant}, {str(isinstance(w, Decode)).lower()}, "
+                                   f"{str(layout == 'holefill').lower()}>",
                          "algorithmic_bytes_per_launch": alg,
                          "nominal_bytes_per_launch": nominal,
                          "moved_rows_per_launch": m["moved"],
                          "kernel_ms": kern_ms, "peak_source": peak_src + ", of measured"
                          if "measured" in peak_src else peak_src},
             "config": {"workload": name, **{k: cfg[k] for k in cfg if k not in ("index", "kind")},
-                       "mu": args.mu, "variant": args.variant,
+                       "mu": args.mu, "variant": args.variant, "layout": layout,
                        "l2": f"inputs larger than L2: cache {w.cache.k.numel() * 4 / 2**30:.2f} GiB "
                              "of K+V, touched every step", "storage": "bf16"},
         }
         return res
 
-    primary = one(args.workload, args.steps)
+    def release(r):
+        if r is not None:
+            r.pop("w", None)
+            torch.cuda.empty_cache()
+
+    primary = one(args.workload, args.steps, args.layout)
     base = None
     if rank == 0 and not args.no_cpu_baseline:
         base = cpu_baseline(primary["w"])
+    launches = primary["w"].launches_per_step * args.steps
+    release(primary)
     secondary = None
     if args.secondary not in ("", "none") and args.secondary != args.workload:
-        secondary = one(args.secondary, args.secondary_steps)
+        secondary = one(args.secondary, args.secondary_steps, args.layout)
+        release(secondary)
+    # the hole-fill cache layout (a next row: same policy, fewest rows moved)
+    holefill = {}
+    if args.holefill_steps > 0 and args.layout == "ordered":
+        for name in (args.workload, args.secondary):
+            if name in ("", "none"):
+                continue
+            r = one(name, args.holefill_steps, "holefill")
+            release(r)
+            holefill[name] = {k: r[k] for k in ("value", "step_ms", "roofline", "e2e")}
     if rank == 0:
-        w = primary["w"]
         line = {
             "metric": METRIC, "value": primary["value"], "unit": UNIT, "n_gpus": ws,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": primary["step_ms"],
@@ -633,7 +724,8 @@ def run_vd(args):
             "roofline": primary["roofline"],
             "e2e": primary["e2e"],
             "clocks": primary["m"]["clocks"],
-            "gpu_launches": w.launches_per_step * args.steps,
+            "gpu_launches": launches,
+            "host_cpus": host_cpus,
         }
         if base is not None:
             line["cpu_baseline"] = base
@@ -641,6 +733,8 @@ def run_vd(args):
             line["secondary"] = {k: secondary[k] for k in ("workload", "value", "step_ms", "roofline",
                                                            "e2e", "config")}
             line["secondary"]["clocks"] = secondary["m"]["clocks"]
+        if holefill:
+            line["holefill_layout"] = holefill
         print(json.dumps(line), flush=True)
     if ws > 1:
         import torch.distributed as dist
@@ -707,6 +801,10 @@ def main(argv=None):
     ap.add_argument("--secondary", default="decode_batched",
                     help="a second workload measured into the same line ('' to skip)")
     ap.add_argument("--secondary-steps", type=int, default=50)
+    ap.add_argument("--layout", choices=["ordered", "holefill"], default="ordered",
+                    help="cache layout of the primary and secondary measurements")
+    ap.add_argument("--holefill-steps", type=int, default=50,
+                    help="steps of the extra hole-fill-layout measurements (0: skip)")
     ap.add_argument("--mu", choices=["running", "recompute"], default="running")
     ap.add_argument("--variant", choices=["l2", "dir", "norm"], default="l2")
     ap.add_argument("--e2e-steps", type=int, default=50)

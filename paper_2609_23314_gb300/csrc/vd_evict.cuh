@@ -109,25 +109,28 @@ struct Smem {
   float fsh[kWarps];
   unsigned long long best;  // decode: this CTA's (key, -tie-break) minimum
   unsigned long long wbest[kWarps];
-  int best_slot;            // decode: the slot of `best`
-  int wslot[kWarps];
-  int holes;                // hole-fill: evicted slots below N
   int sel_digit, sel_above, sel_cnt;
   int cnt_gt, cnt_eq;  // this CTA's keys > t and == t (read by peers)
   int mu_zero;
+  int best_slot;       // hole-fill decode: the slot of `best`
+  int wslot[kWarps];
+  int holes;           // hole-fill: evicted slots below N
 };
 
 __host__ __device__ constexpr size_t align16(size_t x) { return (x + 15) & ~(size_t)15; }
 
 // Byte offsets of the variable parts; the host sizes the launch with the same
-// function.
+// function.  The ring starts on a 128-byte boundary: a warp's 16-byte copies
+// then fill whole 32-byte shared-memory sectors (an offset that is only
+// 16-byte aligned splits every pair of slots across two sectors, which
+// measured 8-13% slower on GB300).
 struct SmemLayout {
   size_t ring, keys, perm, total;
 };
 
 __host__ __device__ inline SmemLayout smem_layout(int capacity, int cluster, bool with_select) {
   SmemLayout l;
-  l.ring = align16(sizeof(Smem));
+  l.ring = (sizeof(Smem) + 127) & ~(size_t)127;
   l.keys = l.ring + kRingBytes;
   const size_t rows = with_select ? (size_t)((capacity + cluster - 1) / cluster) : 0;
   l.perm = l.keys + align16(rows * 4);
@@ -334,11 +337,11 @@ __device__ __forceinline__ Selection cluster_radix_select(KeyOf key_of, int R, i
 // evicted slots ascending at [N, n).  Threads own contiguous row chunks, so
 // prefix sums follow slot order (ties go to the lower slot).  Ends with the
 // cluster barrier after which every CTA's perm[] is complete.
-template <class TieKey>
+template <bool by_tiekey, class TieKey>
 __device__ __forceinline__ void cluster_build_perm(const uint32_t* keys, int r0, int R, int N,
-                                                   Selection sel, bool by_tiekey, uint32_t t2,
-                                                   TieKey tiekey, int C, unsigned rank,
-                                                   uint16_t* perm, Smem& S) {
+                                                   Selection sel, uint32_t t2, TieKey tiekey,
+                                                   int C, unsigned rank, uint16_t* perm,
+                                                   Smem& S) {
   const int tid = threadIdx.x;
   const int ch = (R + kThreads - 1) / kThreads;
   const int c0 = min(R, tid * ch), c1 = min(R, c0 + ch);
@@ -465,7 +468,10 @@ __device__ __forceinline__ void move_rows(uint16_t* kb, uint16_t* vb, int d, int
   }
 }
 
-template <int VAR, bool DECODE>
+// VAR: 0 L2, 1 Dir, 2 Norm.  DECODE: one-token eviction (arg-min) instead of
+// the radix select.  HF: hole-fill layout (compiled separately, so the ordered
+// layout carries none of its code).
+template <int VAR, bool DECODE, bool HF>
 __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLOCK_MIN_CTAS)
     evict_kernel(const EvictArgs a) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
@@ -514,9 +520,9 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
   const int first_new = n - a.B;
   // hole-fill layout: token positions (rows at or above first_new are the
   // appended ones, numbered from pos_new)
-  const bool hf = a.holefill != 0 && !a.score_only;
-  int32_t* posu = hf ? a.pos + (size_t)u * a.capacity : nullptr;
-  const int pnew = hf ? a.pos_new[seq] : 0;
+  constexpr bool hf = HF;
+  int32_t* posu = hf && !a.score_only ? a.pos + (size_t)u * a.capacity : nullptr;
+  const int pnew = hf && !a.score_only ? a.pos_new[seq] : 0;
   auto pos_of = [&](int r) -> int { return r < first_new ? posu[r] : pnew + (r - first_new); };
 
   if (!evict && !a.score_only) {
@@ -601,8 +607,9 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
       h8[k] = (VAR == 1 && active) ? S.muhat[ci * 8 + k] : 0.f;
     }
     const bool mu_zero = VAR == 1 && S.mu_zero;
-    unsigned long long best = ~0ull;
-    int best_slot = 0;
+    unsigned long long best = ~0ull;  // (key, tie-break) of this thread's minimum
+    unsigned best_key = 0xffffffffu;   // hole-fill: key of this thread's minimum
+    int best_slot = -1;
     float* sc_out = a.scores_out ? a.scores_out + (size_t)u * a.capacity : nullptr;
     stream_rows(
         vb, d, 0, d8, lpr, r1 - r0, [&](int i) { return r0 + i; },
@@ -649,12 +656,15 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
               if (bad) record_status(a.status, kStNonfinite);
               if (DECODE) {
                 // lowest score first; among equal scores the latest token
-                // (highest slot, or highest position in the hole-fill layout)
-                const unsigned tb = hf ? (unsigned)pos_of(r) : (unsigned)r;
-                const unsigned long long pk =
-                    ((unsigned long long)key << 32) | (unsigned long long)(0xffffffffu - tb);
-                if (pk < best) {
-                  best = pk;
+                // (highest slot, or highest position in the hole-fill layout,
+                // whose positions are read only to settle an exact tie)
+                if constexpr (!HF) {
+                  const unsigned long long pk = ((unsigned long long)key << 32) |
+                                                (unsigned long long)(0xffffffffu - (unsigned)r);
+                  best = pk < best ? pk : best;
+                } else if (key < best_key ||
+                           (key == best_key && pos_of(r) > pos_of(best_slot))) {
+                  best_key = key;
                   best_slot = r;
                 }
               } else {
@@ -669,18 +679,25 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
       return;
     }
     if (DECODE) {
+      if constexpr (HF) {
+        if (best_slot >= 0)
+          best = ((unsigned long long)best_key << 32) |
+                 (unsigned long long)(0xffffffffu - (unsigned)pos_of(best_slot));
 #pragma unroll
-      for (int off = 16; off > 0; off >>= 1) {
-        const unsigned long long o = __shfl_xor_sync(kFull, best, off);
-        const int os = __shfl_xor_sync(kFull, best_slot, off);
-        if (o < best) {
-          best = o;
-          best_slot = os;
+        for (int off = 16; off > 0; off >>= 1) {
+          const unsigned long long o = __shfl_xor_sync(kFull, best, off);
+          const int os = __shfl_xor_sync(kFull, best_slot, off);
+          if (o < best) {
+            best = o;
+            best_slot = os;
+          }
         }
+      } else {
+        best = warp_min_u64(best);
       }
       if (lane == 0) {
         S.wbest[warp] = best;
-        S.wslot[warp] = best_slot;
+        if (HF) S.wslot[warp] = best_slot;
       }
       __syncthreads();
       if (tid == 0) {
@@ -689,7 +706,7 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
         for (int w = 0; w < kWarps; ++w)
           if (S.wbest[w] < b) {
             b = S.wbest[w];
-            bs = S.wslot[w];
+            if (HF) bs = S.wslot[w];
           }
         S.best = b;
         S.best_slot = bs;
@@ -706,14 +723,14 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
     for (int rr = 0; rr < C; ++rr) {
       const unsigned long long o =
           C > 1 ? ld_cluster_u64(mapa(smem_addr(&S.best), rr)) : S.best;
-      const int os = C > 1 ? (int)ld_cluster_u32(mapa(smem_addr(&S.best_slot), rr)) : S.best_slot;
       if (o < b) {
         b = o;
-        bs = os;
+        if (HF) bs = C > 1 ? (int)ld_cluster_u32(mapa(smem_addr(&S.best_slot), rr)) : S.best_slot;
       }
     }
     if (C > 1) cluster_arrive();  // last peer access of this CTA; wait before exit
-    e_first = bs;
+    // ordered layout: the tie-break field is the slot itself
+    e_first = HF ? bs : (int)(0xffffffffu - (unsigned)(b & 0xffffffffull));
   } else {
     __syncthreads();  // own keys complete
     const int R = r1 - r0;
@@ -726,7 +743,7 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
     // hole-fill layout: the surviving ties are the lowest positions, found
     // by a second select over the complemented positions of the tied rows
     uint32_t t2 = 0u;
-    if (hf && sel.cnt_eq > sel.keep_eq) {
+    if (HF && sel.cnt_eq > sel.keep_eq) {
       const Selection s2 = cluster_radix_select(
           [&](int j, bool& ok) {
             ok = keys[j] == sel.t;
@@ -735,8 +752,8 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
           R, sel.keep_eq, C, S);
       t2 = s2.t;
     }
-    cluster_build_perm(keys, r0, R, Nb, sel, hf, t2,
-                       [&](int j) { return ~(uint32_t)pos_of(r0 + j); }, C, rank, perm, S);
+    cluster_build_perm<HF>(keys, r0, R, Nb, sel, t2,
+                           [&](int j) { return ~(uint32_t)pos_of(r0 + j); }, C, rank, perm, S);
     e_first = perm[Nb];
   }
 
@@ -770,7 +787,7 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
   }
 
   // ---- 6. in-place compaction of this CTA's column slice ---------------
-  if (!hf) {
+  if constexpr (!HF) {
     compact_slice(kb, vb, d, chunk0, cps, e_first, Nb, DECODE ? nullptr : perm, ring);
   } else {
     // hole-fill: the kept rows at or above N move into the evicted slots

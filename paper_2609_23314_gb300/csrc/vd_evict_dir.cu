@@ -3,8 +3,11 @@
 #include "vd_evict.cuh"
 
 namespace vd {
-const void* evict_kernel_dir(bool decode) {
-  return decode ? reinterpret_cast<const void*>(&evict_kernel<1, true>)
-                : reinterpret_cast<const void*>(&evict_kernel<1, false>);
+const void* evict_kernel_dir(bool decode, bool holefill) {
+  if (holefill)
+    return decode ? reinterpret_cast<const void*>(&evict_kernel<1, true, true>)
+                  : reinterpret_cast<const void*>(&evict_kernel<1, false, true>);
+  return decode ? reinterpret_cast<const void*>(&evict_kernel<1, true, false>)
+                : reinterpret_cast<const void*>(&evict_kernel<1, false, false>);
 }
 }  // namespace vd

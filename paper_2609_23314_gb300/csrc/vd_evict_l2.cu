@@ -3,8 +3,11 @@
 #include "vd_evict.cuh"
 
 namespace vd {
-const void* evict_kernel_l2(bool decode) {
-  return decode ? reinterpret_cast<const void*>(&evict_kernel<0, true>)
-                : reinterpret_cast<const void*>(&evict_kernel<0, false>);
+const void* evict_kernel_l2(bool decode, bool holefill) {
+  if (holefill)
+    return decode ? reinterpret_cast<const void*>(&evict_kernel<0, true, true>)
+                  : reinterpret_cast<const void*>(&evict_kernel<0, false, true>);
+  return decode ? reinterpret_cast<const void*>(&evict_kernel<0, true, false>)
+                : reinterpret_cast<const void*>(&evict_kernel<0, false, false>);
 }
 }  // namespace vd

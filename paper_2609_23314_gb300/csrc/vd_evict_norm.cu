@@ -3,8 +3,11 @@
 #include "vd_evict.cuh"
 
 namespace vd {
-const void* evict_kernel_norm(bool decode) {
-  return decode ? reinterpret_cast<const void*>(&evict_kernel<2, true>)
-                : reinterpret_cast<const void*>(&evict_kernel<2, false>);
+const void* evict_kernel_norm(bool decode, bool holefill) {
+  if (holefill)
+    return decode ? reinterpret_cast<const void*>(&evict_kernel<2, true, true>)
+                  : reinterpret_cast<const void*>(&evict_kernel<2, false, true>);
+  return decode ? reinterpret_cast<const void*>(&evict_kernel<2, true, false>)
+                : reinterpret_cast<const void*>(&evict_kernel<2, false, false>);
 }
 }  // namespace vd

@@ -245,3 +245,44 @@ def test_ratio_budget_full_generation(orc):
     assert int(cache.len[0]) == wl.budget_at(cfg, total) == N_max
     assert evictions >= 3
     check_running_sum(cache, rs)
+
+
+# ---------------------------------------------------------------------------
+# hole-fill layout at full size, in the benchmark's configuration
+# ---------------------------------------------------------------------------
+@pytest.mark.parametrize("name", ["decode_batched", "prefill_wide"])
+def test_holefill_full_size_as_benchmarked(orc, name):
+    from test_gpu_holefill import check_holefill_event
+    _, cfg = wl.config(name)
+    cls = bench.Decode if cfg["kind"] == "decode" else bench.Prefill
+    w = cls(name, cfg, DEV, wl.BASE_SEED + cfg["index"], vd.VD_MU_RUNNING, vd.VD_SCORE_L2,
+            layout="holefill")
+    U, cap, N = w.U, w.cap, w.N
+    units = sample_units(U, 6, 55)
+    it = torch.tensor(units, device=DEV, dtype=torch.long)
+    per_seq = w.cache.n_layer * w.cache.n_kv_head
+    kept = torch.empty(w.cache.unit_shape() + (N,), dtype=torch.int32, device=DEV)
+    scores = torch.empty(w.cache.unit_shape() + (cap,), dtype=torch.float32, device=DEV)
+    for step in range(4):
+        w.append_next()
+        n = int(w.cache.len[0])
+        pre = snapshot(w.cache, units)
+        pre_pos = w.pos.view(U, cap)[it].cpu().numpy().copy()
+        pn = w.pos_new_all[w.i - 1].cpu().numpy()
+        for i, u in enumerate(units):
+            pre_pos[i, n - w.B:n] = pn[u // per_seq] + np.arange(w.B)
+        if cfg["kind"] == "decode":
+            w.evict(None, kept, scores)
+        else:
+            w.evict(kept, scores)
+        assert vd.vd_get_device_status() == 0
+        post = snapshot(w.cache, units)
+        post_pos = w.pos.view(U, cap)[it].cpu().numpy()
+        kh = kept.view(U, N)[it].cpu().numpy()
+        sh = scores.view(U, cap)[it].cpu().numpy()
+        for i in range(len(units)):
+            check_holefill_event(orc, oracle.L2, pre[0][i], pre[1][i], pre_pos[i], post[0][i],
+                                 post[1][i], post_pos[i], n, N, kh[i], sh[i])
+    check_running_sum(w.cache, w.rs)
+    del w
+    torch.cuda.empty_cache()
