@@ -56,6 +56,10 @@ def _bind(lib: ctypes.CDLL) -> ctypes.CDLL:
     lib.vdo_mean.restype = None
     lib.vdo_scores.argtypes = [p, i64, i64, ctypes.c_int, p]
     lib.vdo_scores.restype = None
+    lib.vdo_scores_weighted.argtypes = [p, i64, i64, ctypes.c_int, p, p]
+    lib.vdo_scores_weighted.restype = None
+    lib.vdo_dispersion.argtypes = [p, i64, i64]
+    lib.vdo_dispersion.restype = ctypes.c_double
     lib.vdo_select_top_n.argtypes = [p, i64, i64, p]
     lib.vdo_select_top_n.restype = i64
     lib.vdo_evict_unit.argtypes = [p, p, i64, i64, i64, ctypes.c_int, p, p]
@@ -106,6 +110,21 @@ class Oracle:
         out = np.empty(n, np.float64)
         self.lib.vdo_scores(self._ptr(v), n, d, int(variant), self._ptr(out))
         return out
+
+    def scores_weighted(self, v, a, variant: int = L2) -> np.ndarray:
+        """App. A Eq. (app_fastcaote): a_j / (1 - a_j) * s_j."""
+        v = self._u16(v)
+        n, d = v.shape
+        a = np.ascontiguousarray(a, dtype=np.float64)
+        out = np.empty(n, np.float64)
+        self.lib.vdo_scores_weighted(self._ptr(v), n, d, int(variant), self._ptr(a), self._ptr(out))
+        return out
+
+    def dispersion(self, x) -> float:
+        """Sec. 3.1: std over tokens of ||x_i - mean|| (population)."""
+        x = self._u16(x)
+        n, d = x.shape
+        return float(self.lib.vdo_dispersion(self._ptr(x), n, d))
 
     # -- Eq. (eviction) ---------------------------------------------------
     def select_top_n(self, scores, N: int) -> np.ndarray:

@@ -96,6 +96,39 @@ void vdo_scores(const uint16_t* v, int64_t n, int64_t d, int variant, double* ou
   free(mean);
 }
 
+/* App. A, Eq. (app_fastcaote): FastCAOTE evaluates the renormalisation
+ * identity at an observed attention vector and replaces the attention output
+ * by the cache mean, which leaves a_j / (1 - a_j) times the distance from the
+ * mean. */
+void vdo_scores_weighted(const uint16_t* v, int64_t n, int64_t d, int variant, const double* a,
+                         double* out) {
+  vdo_scores(v, n, d, variant, out);
+  for (int64_t j = 0; j < n; ++j) {
+    if (a[j] >= 0.0 && a[j] < 1.0)
+      out[j] *= a[j] / (1.0 - a[j]);
+    else
+      out[j] = NAN;
+  }
+}
+
+/* Sec. 3.1: the standard deviation over tokens of the L2 distance from the
+ * cache mean (divisor n), from a compensated two-pass computation. */
+double vdo_dispersion(const uint16_t* x, int64_t n, int64_t d) {
+  double* s = (double*)malloc((size_t)n * sizeof(double));
+  vdo_scores(x, n, d, VDO_L2, s);
+  double sum = 0.0, corr = 0.0;
+  for (int64_t j = 0; j < n; ++j) {
+    double t = sum + s[j];
+    corr += fabs(sum) >= fabs(s[j]) ? (sum - t) + s[j] : (s[j] - t) + sum;
+    sum = t;
+  }
+  const double m = (sum + corr) / (double)n;
+  double ss = 0.0;
+  for (int64_t j = 0; j < n; ++j) ss += (s[j] - m) * (s[j] - m);
+  free(s);
+  return sqrt(ss / (double)n);
+}
+
 typedef struct {
   double score;
   int32_t index;

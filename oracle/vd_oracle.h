@@ -43,6 +43,16 @@ void vdo_mean(const uint16_t* v, int64_t n, int64_t d, double* out);
  * DIR with a zero-norm v_j or a zero-norm mean takes cos := 0 (score 1). */
 void vdo_scores(const uint16_t* v, int64_t n, int64_t d, int variant, double* out);
 
+/* App. A, Eq. (app_fastcaote): the attention-weighted score
+ * a_j / (1 - a_j) * s_j, with s_j the `variant` score of vdo_scores and a_j
+ * the caller's attention weight (a_j in [0, 1); outside -> NaN).  out: [n]. */
+void vdo_scores_weighted(const uint16_t* v, int64_t n, int64_t d, int variant, const double* a,
+                         double* out);
+
+/* Sec. 3.1 (and App. C): sigma = std_i || x_i - mean ||_2 over the n rows of
+ * one unit (population standard deviation).  Returns sigma. */
+double vdo_dispersion(const uint16_t* x, int64_t n, int64_t d);
+
 /* Eq. (eviction): keep the N highest scores, ties to the lower index.
  * Writes the kept indices in ascending order to kept[0..min(n,N)).
  * Returns the number kept (min(n, N)); n <= N keeps everything. */

@@ -78,6 +78,18 @@ def golden_cases():
 
 
 def check_golden(orc, case):
+    if "dispersion" in case:
+        x = oracle.bf16_bits(np.asarray(case["x"], np.float32))
+        assert math.isclose(orc.dispersion(x), closed_form(case["dispersion"]), rel_tol=1e-12,
+                            abs_tol=1e-15)
+        return
+    if "weights" in case:
+        v = oracle.bf16_bits(np.asarray(case["v"], np.float32))
+        s = orc.scores_weighted(v, np.asarray(case["weights"], np.float64), oracle.L2)
+        want = np.array([closed_form(x) for x in case["weighted_scores"]])
+        assert np.allclose(s, want, rtol=1e-12, atol=1e-12), (s, want)
+        assert orc.select_top_n(s, case["N"]).tolist() == case["kept"]
+        return
     if "v_stream" in case:
         d_vs = np.asarray(case["v_stream"], np.float32).reshape(-1, 1)
         d_ks = np.asarray(case["k_stream"], np.float32).reshape(-1, 1)
@@ -324,6 +336,38 @@ def check_block_equivalences(orc, rng):
     assert np.array_equal(vc, vv) and np.array_equal(kc, kk)
 
 
+# --------------------------------------------------------------------------
+# App. A, Eq. (app_fastcaote) and (recon_error): the weighted score at the
+# uniform attention vector is the brute-force output disturbance
+# --------------------------------------------------------------------------
+def check_fastcaote_uniform(orc, v):
+    x = as_float(v)
+    n = x.shape[0]
+    w = orc.scores_weighted(v, np.full(n, 1.0 / n), oracle.L2)
+    o_star = x.mean(axis=0)
+    for j in range(n):                       # drop token j, renormalise uniformly
+        o_minus_j = np.delete(x, j, axis=0).mean(axis=0)
+        assert math.isclose(w[j], np.linalg.norm(o_star - o_minus_j), rel_tol=1e-10,
+                            abs_tol=1e-12)
+    # zero attention weight -> zero score; the uniform ranking is ValueDiff's
+    z = np.full(n, 1.0 / n)
+    z[0] = 0.0
+    assert orc.scores_weighted(v, z, oracle.L2)[0] == 0.0
+    assert np.array_equal(orc.select_top_n(w, n // 2),
+                          orc.select_top_n(orc.scores(v, oracle.L2), n // 2))
+
+
+# --------------------------------------------------------------------------
+# Sec. 3.1: sigma = std over tokens of the distance from the cache mean
+# --------------------------------------------------------------------------
+def check_dispersion(orc, x_bits):
+    x = as_float(x_bits)
+    dist = np.linalg.norm(x - x.mean(axis=0), axis=1)
+    assert math.isclose(orc.dispersion(x_bits), float(np.std(dist)), rel_tol=1e-10, abs_tol=1e-12)
+    same = np.repeat(x_bits[:1], 5, axis=0)
+    assert orc.dispersion(same) == 0.0
+
+
 def all_checks(orc, seed=0):
     """Every pin at a small size; returns the list of (name, error) failures."""
     rng = np.random.default_rng(seed)
@@ -353,5 +397,7 @@ def all_checks(orc, seed=0):
     for var in (oracle.L2, oracle.DIR, oracle.NORM):
         run(f"gather:{var}", check_gather, orc, rng, 37, 8, 20, var)
     run("special_cases", check_special_cases, orc, rng)
+    run("fastcaote_uniform", check_fastcaote_uniform, orc, gauss_cache(rng, 9, 6))
+    run("dispersion", check_dispersion, orc, gauss_cache(rng, 40, 8))
     run("block_equivalences", check_block_equivalences, orc, rng)
     return failures

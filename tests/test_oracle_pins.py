@@ -111,3 +111,19 @@ def test_sum_rows_is_exact_for_bf16(orc):
     for c in range(4):
         exact = sum(Fraction(float(t)) for t in x[:, c])
         assert got[c] == float(exact)
+
+
+@pytest.mark.parametrize("n,d", [(2, 3), (7, 5), (16, 8)])
+def test_fastcaote_at_uniform_attention(orc, n, d):
+    pins.check_fastcaote_uniform(orc, pins.gauss_cache(np.random.default_rng(n * 31 + d), n, d))
+
+
+@pytest.mark.parametrize("n,d", [(3, 1), (50, 16), (400, 64)])
+def test_dispersion_definition(orc, n, d):
+    pins.check_dispersion(orc, pins.gauss_cache(np.random.default_rng(n + 2 * d), n, d))
+
+
+def test_weights_outside_unit_interval_give_nan(orc):
+    v = pins.gauss_cache(np.random.default_rng(1), 4, 4)
+    s = orc.scores_weighted(v, np.array([0.2, 1.0, -0.1, 0.0]), oracle.L2)
+    assert np.isnan(s[1]) and np.isnan(s[2]) and s[3] == 0.0 and s[0] > 0

@@ -39,6 +39,10 @@ MUTANTS = {
     # V gathered from K's rows (transposed operand)
     "gather_wrong_tensor": ("memcpy(vv + r * d, v + (int64_t)idx[r] * d, row_bytes);",
                             "memcpy(vv + r * d, k + (int64_t)idx[r] * d, row_bytes);"),
+    # FastCAOTE factor a/(1+a) instead of a/(1-a)
+    "weight_factor": ("out[j] *= a[j] / (1.0 - a[j]);", "out[j] *= a[j] / (1.0 + a[j]);"),
+    # sample standard deviation instead of the population one
+    "dispersion_divisor": ("return sqrt(ss / (double)n);", "return sqrt(ss / (double)(n - 1));"),
     # gather off by one row
     "gather_off_by_one": ("memcpy(kk + r * d, k + (int64_t)idx[r] * d, row_bytes);",
                           "memcpy(kk + r * d, k + (int64_t)(idx[r] > 0 ? idx[r] - 1 : 0) * d, row_bytes);"),
