@@ -135,6 +135,37 @@ vd_status vd_evict_decode(const vd_cache* c, int32_t N, const int32_t* N_dev, vd
                           vd_mu_mode mu, double* running_sum, int32_t* evicted_out,
                           int32_t* kept_idx_out, float* scores_out, vd_stream_t stream);
 
+/* Scores with options, no eviction.
+ *   score_keys      0: V rows (ValueDiff and its variants, Sec. 3.2); 1: the
+ *                   same rules on K rows, with the mean of K (the key-side
+ *                   signals of the Sec. 4 baselines: L2 = distance from the key
+ *                   centroid, Dir = cosine distance from the mean key).
+ *   scores_out      nullable fp32 [..][capacity] (rows >= len untouched).
+ *   dispersion_out  nullable fp32 [n_seq][n_layer][n_kv_head]: per unit, the
+ *                   standard deviation over its len tokens of the L2 distance
+ *                   from the mean -- sigma_V (or sigma_K with score_keys) of
+ *                   Sec. 3.1 (population std).  Requires var == VD_SCORE_L2.
+ * At least one of the two outputs must be given.  The mean is recomputed. */
+vd_status vd_score_ex(const vd_cache* c, vd_variant var, int32_t score_keys, float* scores_out,
+                      float* dispersion_out, vd_stream_t stream);
+
+/* vd_evict_block with scoring options:
+ *   score_keys  1: select on the K-side rule (mean of K); only with
+ *               VD_MU_RECOMPUTE (the running sum tracks V) -> else
+ *               VD_ERR_UNSUPPORTED.  K and V are still both compacted.
+ *   attn        nullable fp32 device [..][capacity]: an attention weight a_j
+ *               in [0, 1) per cached token; the score becomes
+ *               a_j / (1 - a_j) * s_j, the FastCAOTE form of App. A
+ *               Eq. (app_fastcaote) (with VD_SCORE_L2).  A weight outside
+ *               [0, 1) gives a NaN score (ranked lowest, VD_ERR_NONFINITE).
+ *               scores_out then holds the weighted scores.
+ * Other arguments as in vd_evict_block.  A weighted decode step is this call
+ * with B = 1. */
+vd_status vd_evict_block_ex(const vd_cache* c, int32_t N, const int32_t* N_dev, int32_t B,
+                            vd_variant var, vd_mu_mode mu, double* running_sum,
+                            int32_t score_keys, const float* attn, int32_t* kept_idx_out,
+                            float* scores_out, vd_stream_t stream);
+
 /* Hole-fill layout (not in the paper; its eviction rule with a cache layout
  * that moves as few rows as possible).  Same policy as vd_evict_block /
  * vd_evict_decode (Sec. 2.1, Eq. eviction; Sec. 2.2, Eq. block_processing),

@@ -20,7 +20,8 @@ import threading
 
 __all__ = [
     "VD_SCORE_L2", "VD_SCORE_DIR", "VD_SCORE_NORM", "VD_MU_RECOMPUTE", "VD_MU_RUNNING",
-    "VdError", "Cache", "vd_score", "vd_evict_block", "vd_evict_decode",
+    "VdError", "Cache", "vd_score", "vd_score_ex", "vd_evict_block", "vd_evict_block_ex",
+    "vd_evict_decode",
     "vd_evict_block_holefill", "vd_evict_decode_holefill", "vd_append",
     "vd_running_sum_init", "vd_workspace_size", "vd_status_string", "vd_get_device_status",
     "library_path", "load_library",
@@ -69,6 +70,8 @@ def load_library() -> ctypes.CDLL:
             lib.vd_evict_decode.argtypes = [cp, I32, P, S, S, P, P, P, P, P]
             lib.vd_evict_block_holefill.argtypes = [cp, I32, P, I32, S, S, P, P, P, P, P, P]
             lib.vd_evict_decode_holefill.argtypes = [cp, I32, P, S, S, P, P, P, P, P, P, P]
+            lib.vd_score_ex.argtypes = [cp, S, I32, P, P, P]
+            lib.vd_evict_block_ex.argtypes = [cp, I32, P, I32, S, S, P, I32, P, P, P, P]
             lib.vd_append.argtypes = [cp, P, P, I32, P]
             lib.vd_running_sum_init.argtypes = [cp, P, P]
             lib.vd_workspace_size.argtypes = [cp]
@@ -76,7 +79,8 @@ def load_library() -> ctypes.CDLL:
             lib.vd_status_string.argtypes = [S]
             lib.vd_status_string.restype = ctypes.c_char_p
             lib.vd_get_device_status.argtypes = [P]
-            for f in ("vd_score", "vd_evict_block", "vd_evict_decode", "vd_evict_block_holefill",
+            for f in ("vd_score", "vd_score_ex", "vd_evict_block_ex", "vd_evict_block",
+                      "vd_evict_decode", "vd_evict_block_holefill",
                       "vd_evict_decode_holefill", "vd_append", "vd_running_sum_init",
                       "vd_get_device_status"):
                 getattr(lib, f).restype = S
@@ -199,6 +203,36 @@ def vd_evict_decode(cache: Cache, N: int, N_dev=None, variant: int = VD_SCORE_L2
     _check(load_library().vd_evict_decode(cache.ref(), int(N), args[0], int(variant), int(mu),
                                           args[1], args[2], args[3], args[4], _stream(stream)),
            "vd_evict_decode")
+
+
+def vd_score_ex(cache: Cache, variant: int, score_keys: bool = False, scores_out=None,
+                dispersion_out=None, stream=None) -> None:
+    """Scores of V (or K) rows and/or the per-unit dispersion sigma."""
+    torch = _torch()
+    us = cache.unit_shape()
+    sc = _ptr(scores_out, torch.float32, us + (cache.capacity,), "scores_out", cache.device)
+    dp = _ptr(dispersion_out, torch.float32, us, "dispersion_out", cache.device)
+    _check(load_library().vd_score_ex(cache.ref(), int(variant), int(bool(score_keys)), sc, dp,
+                                      _stream(stream)), "vd_score_ex")
+
+
+def vd_evict_block_ex(cache: Cache, N: int, N_dev=None, B: int = 0, variant: int = VD_SCORE_L2,
+                      mu: int = VD_MU_RECOMPUTE, running_sum=None, score_keys: bool = False,
+                      attn=None, kept_idx_out=None, scores_out=None, stream=None) -> None:
+    """Block eviction on the K-side rule and/or with attention weights."""
+    torch = _torch()
+    us = cache.unit_shape()
+    args = (
+        _ptr(N_dev, torch.int32, (cache.n_seq,), "N_dev", cache.device),
+        _ptr(running_sum, torch.float64, us + (cache.head_dim,), "running_sum", cache.device),
+        _ptr(attn, torch.float32, us + (cache.capacity,), "attn", cache.device),
+        _ptr(kept_idx_out, torch.int32, us + (int(N),), "kept_idx_out", cache.device),
+        _ptr(scores_out, torch.float32, us + (cache.capacity,), "scores_out", cache.device),
+    )
+    _check(load_library().vd_evict_block_ex(cache.ref(), int(N), args[0], int(B), int(variant),
+                                            int(mu), args[1], int(bool(score_keys)), args[2],
+                                            args[3], args[4], _stream(stream)),
+           "vd_evict_block_ex")
 
 
 def vd_evict_block_holefill(cache: Cache, N: int, pos, pos_first_new, N_dev=None, B: int = 0,

@@ -265,7 +265,8 @@ vd_status launch(const void* kern, long long units, int c, size_t smem, const vd
 vd_status run(const vd_cache* c, int32_t N, const int32_t* N_dev, int32_t B, vd_variant var,
               vd_mu_mode mu, double* running_sum, int32_t* evicted_out, int32_t* kept_idx_out,
               float* scores_out, cudaStream_t s, bool decode, bool score_only,
-              int32_t* pos = nullptr, const int32_t* pos_new = nullptr) {
+              int32_t* pos = nullptr, const int32_t* pos_new = nullptr, int score_k = 0,
+              const float* weights = nullptr, float* disp_out = nullptr) {
   vd_status r = validate_cache(c);
   if (r != VD_OK) return r;
   if (var != VD_SCORE_L2 && var != VD_SCORE_DIR && var != VD_SCORE_NORM) return VD_ERR_INVALID_ARG;
@@ -274,9 +275,12 @@ vd_status run(const vd_cache* c, int32_t N, const int32_t* N_dev, int32_t B, vd_
     if (N < 1 || N > c->capacity) return VD_ERR_INVALID_ARG;
     if (B < 0 || B > c->capacity) return VD_ERR_INVALID_ARG;
     if (mu == VD_MU_RUNNING && !running_sum) return VD_ERR_INVALID_ARG;
-  } else if (!scores_out) {
+  } else if (!scores_out && !disp_out) {
     return VD_ERR_INVALID_ARG;
   }
+  if (disp_out && (!score_only || var != VD_SCORE_L2)) return VD_ERR_INVALID_ARG;
+  if (weights && (score_only || decode)) return VD_ERR_INVALID_ARG;
+  if (score_k && mu == VD_MU_RUNNING && !score_only) return VD_ERR_UNSUPPORTED;
   const bool holefill = pos != nullptr || pos_new != nullptr;
   if (holefill && (!pos || !pos_new)) return VD_ERR_INVALID_ARG;
   DeviceState* st = nullptr;
@@ -312,6 +316,9 @@ vd_status run(const vd_cache* c, int32_t N, const int32_t* N_dev, int32_t B, vd_
   a.pos = pos;
   a.pos_new = pos_new;
   a.holefill = holefill ? 1 : 0;
+  a.score_k = score_k ? 1 : 0;
+  a.weights = weights;
+  a.disp_out = disp_out;
   size_t smem = 0;
   a.cluster = choose_cluster(kern, units, c->head_dim, c->capacity, !small, *st, &smem);
   if (smem > (size_t)st->smem_optin) return VD_ERR_UNSUPPORTED;
@@ -349,6 +356,22 @@ vd_status vd_evict_decode(const vd_cache* c, int32_t N, const int32_t* N_dev, vd
                           int32_t* kept_idx_out, float* scores_out, vd_stream_t stream) {
   return run(c, N, N_dev, 1, var, mu, running_sum, evicted_out, kept_idx_out, scores_out,
              reinterpret_cast<cudaStream_t>(stream), true, false);
+}
+
+vd_status vd_score_ex(const vd_cache* c, vd_variant var, int32_t score_keys, float* scores_out,
+                      float* dispersion_out, vd_stream_t stream) {
+  return run(c, 1, nullptr, 0, var, VD_MU_RECOMPUTE, nullptr, nullptr, nullptr, scores_out,
+             reinterpret_cast<cudaStream_t>(stream), false, true, nullptr, nullptr, score_keys,
+             nullptr, dispersion_out);
+}
+
+vd_status vd_evict_block_ex(const vd_cache* c, int32_t N, const int32_t* N_dev, int32_t B,
+                            vd_variant var, vd_mu_mode mu, double* running_sum,
+                            int32_t score_keys, const float* attn, int32_t* kept_idx_out,
+                            float* scores_out, vd_stream_t stream) {
+  return run(c, N, N_dev, B, var, mu, running_sum, nullptr, kept_idx_out, scores_out,
+             reinterpret_cast<cudaStream_t>(stream), false, false, nullptr, nullptr, score_keys,
+             attn, nullptr);
 }
 
 vd_status vd_evict_block_holefill(const vd_cache* c, int32_t N, const int32_t* N_dev, int32_t B,

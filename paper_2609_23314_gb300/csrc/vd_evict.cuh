@@ -92,6 +92,9 @@ struct EvictArgs {
   int32_t* pos;            // hole-fill layout: token positions [U][capacity]
   const int32_t* pos_new;  // hole-fill layout: position of row len - B, [n_seq]
   int32_t holefill;        // 1: hole-fill layout (ties by position), 0: ordered
+  int32_t score_k;         // 1: mean and scores from K (key-side rules)
+  const float* weights;    // nullable [U][capacity]: attention weights a_j (block path)
+  float* disp_out;         // nullable [U]: std of the L2 scores (score-only path)
 };
 
 // Fixed part of the dynamic shared memory.  After it (16-byte aligned): the
@@ -115,6 +118,7 @@ struct Smem {
   int best_slot;       // hole-fill decode: the slot of `best`
   int wslot[kWarps];
   int holes;           // hole-fill: evicted slots below N
+  float disp[4];       // dispersion partials: sum s (hi, lo), sum s^2 (hi, lo)
 };
 
 __host__ __device__ constexpr size_t align16(size_t x) { return (x + 15) & ~(size_t)15; }
@@ -493,6 +497,7 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
   const size_t ubase = (size_t)u * a.capacity * d;
   uint16_t* kb = a.k + ubase;
   uint16_t* vb = a.v + ubase;
+  const uint16_t* sb = a.score_k ? kb : vb;  // rows the mean and the scores come from
 
   // ---- validation: uniform across the cluster (per-sequence values only) ---
   if (n < 0 || n > a.capacity || (a.mu_running && !a.score_only && a.B > n)) {
@@ -560,7 +565,7 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
       p0 = r0;
       p1 = r1;
     }
-    sum_rows(vb, d, 0, d8, lpr, max(0, p1 - p0), [&](int i) { return p0 + i; },
+    sum_rows(sb, d, 0, d8, lpr, max(0, p1 - p0), [&](int i) { return p0 + i; },
              [](int) { return 1.f; }, S, ring);
     if (C > 1) cluster_sync(); else __syncthreads();
     if (tid < d) {
@@ -607,12 +612,15 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
       h8[k] = (VAR == 1 && active) ? S.muhat[ci * 8 + k] : 0.f;
     }
     const bool mu_zero = VAR == 1 && S.mu_zero;
+    const bool weighted = !DECODE && a.weights != nullptr;
+    const bool disp = a.score_only && a.disp_out != nullptr;
+    float ds_hi = 0.f, ds_lo = 0.f, dq_hi = 0.f, dq_lo = 0.f;  // dispersion sums
     unsigned long long best = ~0ull;  // (key, tie-break) of this thread's minimum
     unsigned best_key = 0xffffffffu;   // hole-fill: key of this thread's minimum
     int best_slot = -1;
     float* sc_out = a.scores_out ? a.scores_out + (size_t)u * a.capacity : nullptr;
     stream_rows(
-        vb, d, 0, d8, lpr, r1 - r0, [&](int i) { return r0 + i; },
+        sb, d, 0, d8, lpr, r1 - r0, [&](int i) { return r0 + i; },
         [&](int item, bool in, const uint4& q) {
           float x[8];
           unpack8(q, x);
@@ -649,7 +657,13 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
           }
           if (in && ci == 0) {
             const int r = r0 + item;
-            if (sc_out) sc_out[r] = s;
+            if (sc_out && !weighted) sc_out[r] = s;
+            if (disp) {  // sum s and s^2 (the square split exactly by an FMA)
+              ff_accumulate(ds_hi, ds_lo, s);
+              const float q2 = s * s;
+              ff_accumulate(dq_hi, dq_lo, q2);
+              dq_lo += fmaf(s, s, -q2);
+            }
             if (!a.score_only) {
               bool bad;
               const uint32_t key = score_key(s, bad);
@@ -676,6 +690,52 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
         ring);
     if (a.score_only) {
       if (score_split) cluster_wait();
+      if (disp) {
+        // dispersion of the scores over the unit: std_j s_j = sqrt(E[s^2] - E[s]^2),
+        // the CTA sums merged in a fixed order, then across the cluster
+        ff a1 = ff_add(ff{ds_hi, 0.f}, ff{0.f, ds_lo});
+        ff a2 = ff_add(ff{dq_hi, 0.f}, ff{0.f, dq_lo});
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) {
+          a1 = ff_add(a1, ff_shfl_xor(a1, off));
+          a2 = ff_add(a2, ff_shfl_xor(a2, off));
+        }
+        if (lane == 0) {
+          S.acc_hi[warp] = a1.hi;
+          S.acc_lo[warp] = a1.lo;
+          S.acc_hi[32 + warp] = a2.hi;
+          S.acc_lo[32 + warp] = a2.lo;
+        }
+        __syncthreads();
+        if (tid == 0) {
+          ff t1{0.f, 0.f}, t2{0.f, 0.f};
+          for (int w = 0; w < kWarps; ++w) {
+            t1 = ff_add(t1, ff{S.acc_hi[w], S.acc_lo[w]});
+            t2 = ff_add(t2, ff{S.acc_hi[32 + w], S.acc_lo[32 + w]});
+          }
+          S.disp[0] = t1.hi;
+          S.disp[1] = t1.lo;
+          S.disp[2] = t2.hi;
+          S.disp[3] = t2.lo;
+        }
+        if (C > 1) cluster_sync(); else __syncthreads();
+        if (rank == 0 && tid == 0) {
+          double s1 = 0.0, s2 = 0.0;
+          for (int rr = 0; rr < C; ++rr) {
+            const uint32_t base = smem_addr(&S.disp[0]);
+            float v[4];
+            for (int k = 0; k < 4; ++k)
+              v[k] = C > 1 ? ld_cluster_f32(mapa(base + 4u * (unsigned)k, (unsigned)rr))
+                           : S.disp[k];
+            s1 += (double)v[0] + (double)v[1];
+            s2 += (double)v[2] + (double)v[3];
+          }
+          const double m = s1 / (double)n;
+          const double var = s2 / (double)n - m * m;
+          a.disp_out[u] = (float)sqrt(var > 0.0 ? var : 0.0);
+        }
+        if (C > 1) cluster_sync();  // peers stay until rank 0 has read them
+      }
       return;
     }
     if (DECODE) {
@@ -734,6 +794,22 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
   } else {
     __syncthreads();  // own keys complete
     const int R = r1 - r0;
+    if (a.weights) {
+      // attention-weighted score (the FastCAOTE form of App. A):
+      // s'_j = a_j / (1 - a_j) * s_j, for weights a_j in [0, 1)
+      const float* wu = a.weights + (size_t)u * a.capacity;
+      float* sc_out = a.scores_out ? a.scores_out + (size_t)u * a.capacity : nullptr;
+      for (int j = tid; j < R; j += kThreads) {
+        const float w = wu[r0 + j];
+        const float f = (w >= 0.f && w < 1.f) ? w / (1.f - w) : __int_as_float(0x7fc00000);
+        const float sw = __uint_as_float(keys[j]) * f;
+        bool bad;
+        keys[j] = score_key(sw, bad);
+        if (bad) record_status(a.status, kStNonfinite);
+        if (sc_out) sc_out[r0 + j] = sw;
+      }
+      __syncthreads();
+    }
     const Selection sel = cluster_radix_select(
         [&](int j, bool& ok) {
           ok = true;

@@ -1,0 +1,160 @@
+"""The scoring options of vd_score_ex / vd_evict_block_ex against the fp64
+oracle: key-side rules (the same scores on K), attention-weighted scores
+(App. A Eq. app_fastcaote) and the per-unit dispersion sigma (Sec. 3.1).
+Needs a GB300."""
+from __future__ import annotations
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import paper_2609_23314_gb300 as vd
+from paper_2609_23314_gb300 import build, workloads as wl
+from vd_gpu import RTOL, bits, near_tie_band, new_cache, score_tolerance, units_view
+
+pytestmark = pytest.mark.gpu
+VARS = [oracle.L2, oracle.DIR, oracle.NORM]
+VAR_IDS = ["l2", "dir", "norm"]
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    build.build()
+    vd.load_library()
+    torch.cuda.set_device(0)
+    yield
+    assert vd.vd_get_device_status() == 0
+
+
+def filled(n_seq, L, H, cap, d, lens, seed, gen="gauss_outlier"):
+    cache = new_cache(n_seq, L, H, cap, d)
+    st = wl.TokenStream(gen, cache.units, d, device="cuda", seed=seed)
+    wl.fill_rows(st, units_view(cache.k), units_view(cache.v), cap)
+    cache.len.copy_(torch.tensor(lens, dtype=torch.int32))
+    return cache
+
+
+def check_scored_event(s_ora, tol, pre_k, pre_v, post_k, post_v, n, N, kept_gpu, scores_gpu):
+    """One unit: GPU scores within tol of the oracle's, the same kept set
+    outside near ties, bit-exact gathers of K and V."""
+    if n <= N:
+        assert np.array_equal(post_v[:n], pre_v[:n]) and np.array_equal(post_k[:n], pre_k[:n])
+        return
+    err = np.abs(scores_gpu[:n].astype(np.float64) - s_ora)
+    assert np.all(err <= tol), f"worst score error {err.max():.3e}"
+    kept_ora = orc_select(s_ora, N)
+    kg = np.asarray(kept_gpu[:N], np.int64)
+    assert np.all(np.diff(kg) > 0)
+    diff = np.setxor1d(kg, kept_ora)
+    if diff.size:
+        assert np.all(near_tie_band(s_ora, N)[diff]), f"kept sets differ at {diff[:8]}"
+    assert np.array_equal(post_k[:N], pre_k[:n][kg]) and np.array_equal(post_v[:N], pre_v[:n][kg])
+
+
+_ORC = None
+
+
+def orc_select(s, N):
+    return _ORC.select_top_n(s, N)
+
+
+def run_ex(orc, cache, N, B, var, score_keys, attn):
+    global _ORC
+    _ORC = orc
+    U, cap = cache.units, cache.capacity
+    per_seq = cache.n_layer * cache.n_kv_head
+    lens = cache.len.cpu().numpy().copy()
+    pre_k, pre_v = bits(units_view(cache.k)), bits(units_view(cache.v))
+    us = cache.unit_shape()
+    kept = torch.full(us + (N,), -7, dtype=torch.int32, device="cuda")
+    scores = torch.full(us + (cap,), float("nan"), device="cuda")
+    vd.vd_evict_block_ex(cache, N, None, B, var, vd.VD_MU_RECOMPUTE, None, score_keys, attn, kept,
+                         scores)
+    assert vd.vd_get_device_status() == 0
+    post_k, post_v = bits(units_view(cache.k)), bits(units_view(cache.v))
+    kh, sh = kept.view(U, N).cpu().numpy(), scores.view(U, cap).cpu().numpy()
+    a_h = attn.view(U, cap).cpu().numpy().astype(np.float64) if attn is not None else None
+    for u in range(U):
+        n = int(lens[u // per_seq])
+        src = pre_k[u, :n] if score_keys else pre_v[u, :n]
+        if a_h is None:
+            s_ora = orc.scores(src, var)
+            tol = score_tolerance(var, s_ora, src, orc.mean(src))
+        else:
+            s_ora = orc.scores_weighted(src, a_h[u, :n], var)
+            base = orc.scores(src, var)
+            f = a_h[u, :n] / (1.0 - a_h[u, :n])
+            # the weight multiplies the score: its error scales with the factor,
+            # plus one fp32 rounding of the product
+            tol = score_tolerance(var, base, src, orc.mean(src)) * f + 2e-7 * np.abs(s_ora)
+        check_scored_event(s_ora, tol, pre_k[u], pre_v[u], post_k[u], post_v[u], n, N, kh[u], sh[u])
+
+
+@pytest.mark.parametrize("var", VARS, ids=VAR_IDS)
+@pytest.mark.parametrize("cluster", [1, 4])
+def test_key_side_eviction(orc, var, cluster, monkeypatch):
+    monkeypatch.setenv("VD_CLUSTER_SIZE", str(cluster))
+    d, N, B = 128, 300, 64
+    cache = filled(3, 2, 2, N + B, d, [N + B, N + 10, 50], seed=17 + cluster)
+    run_ex(orc, cache, N, B, var, True, None)
+
+
+@pytest.mark.parametrize("var", VARS, ids=VAR_IDS)
+@pytest.mark.parametrize("cluster", [1, 2])
+def test_attention_weighted_eviction(orc, var, cluster, monkeypatch):
+    monkeypatch.setenv("VD_CLUSTER_SIZE", str(cluster))
+    d, N, B = 64, 200, 40
+    cache = filled(2, 2, 2, N + B, d, [N + B, N + 7], seed=23 + cluster)
+    g = torch.Generator(device="cuda").manual_seed(5)
+    attn = torch.rand(cache.unit_shape() + (N + B,), generator=g, device="cuda") * 0.9
+    attn[..., ::17] = 0.0                     # tokens with no attention score 0
+    run_ex(orc, cache, N, B, var, False, attn)
+
+
+def test_uniform_attention_keeps_the_valuediff_set(orc):
+    """App. A: with a_j = 1/n the weighted rule ranks like ValueDiff."""
+    d, N, n = 128, 150, 200
+    cache = filled(1, 2, 2, n, d, [n], seed=3)
+    ref = vd.Cache(cache.k.clone(), cache.v.clone(), cache.len.clone())
+    attn = torch.full(cache.unit_shape() + (n,), 1.0 / n, device="cuda")
+    ka = torch.empty(cache.unit_shape() + (N,), dtype=torch.int32, device="cuda")
+    kb = torch.empty_like(ka)
+    vd.vd_evict_block_ex(cache, N, attn=attn, kept_idx_out=ka)
+    vd.vd_evict_block(ref, N, kept_idx_out=kb)
+    assert vd.vd_get_device_status() == 0
+    assert torch.equal(ka, kb)
+
+
+@pytest.mark.parametrize("keys", [False, True], ids=["sigma_v", "sigma_k"])
+@pytest.mark.parametrize("cluster", [1, 2, 4])
+def test_dispersion_matches_oracle(orc, keys, cluster, monkeypatch):
+    monkeypatch.setenv("VD_CLUSTER_SIZE", str(cluster))
+    d = 128
+    lens = [2048, 777, 1]
+    cache = filled(3, 2, 2, 2048, d, lens, seed=41, gen="student_t")
+    out = torch.full(cache.unit_shape(), -1.0, device="cuda")
+    vd.vd_score_ex(cache, vd.VD_SCORE_L2, keys, None, out)
+    assert vd.vd_get_device_status() == 0
+    src = bits(units_view(cache.k if keys else cache.v))
+    got = out.view(-1).cpu().numpy()
+    for u in range(cache.units):
+        n = lens[u // 4]
+        want = orc.dispersion(src[u, :n])
+        assert abs(got[u] - want) <= 1e-5 * want + 1e-6, (u, got[u], want)
+
+
+def test_option_errors():
+    cache = filled(1, 1, 1, 64, 64, [64], seed=1)
+    rs = torch.zeros(1, 1, 1, 64, dtype=torch.float64, device="cuda")
+    with pytest.raises(vd.VdError) as e:
+        vd.vd_evict_block_ex(cache, 32, None, 0, vd.VD_SCORE_L2, vd.VD_MU_RUNNING, rs, True)
+    assert e.value.code == 3                  # the running sum tracks V only
+    with pytest.raises(vd.VdError) as e:
+        vd.vd_score_ex(cache, vd.VD_SCORE_DIR, False, None,
+                       torch.zeros(1, 1, 1, device="cuda"))
+    assert e.value.code == 1                  # sigma is defined on L2 distances
+    attn = torch.full((1, 1, 1, 64), 0.5, device="cuda")
+    attn[..., 3] = 1.0                        # a weight of 1: infinite factor
+    vd.vd_evict_block_ex(cache, 32, attn=attn)
+    assert vd.vd_get_device_status() == 4
