@@ -219,7 +219,8 @@ class ClockSampler:
 class Prefill:
     """Block boundary at steady state: append B rows, evict N + B -> N."""
 
-    def __init__(self, name, cfg, device, seed, mu, variant, n_blocks=8, layout="ordered"):
+    def __init__(self, name, cfg, device, seed, mu, variant, n_blocks=8, layout="ordered",
+                 score_keys=False, weighted=False):
         """n_blocks distinct appended blocks are pre-generated and reused in
         order; the benchmark asks for as many as the prompt has (T / B), so
         every timed event appends rows the cache has not seen.  layout
@@ -258,6 +259,13 @@ class Prefill:
             steps = torch.arange(1 << 14, dtype=torch.int32, device=device)
             self.pos_new_all = (self.N + self.B * steps).view(-1, 1).repeat(
                 1, cfg["n_seq"]).contiguous()
+        # scoring options (key-side rule; attention weights in [0, 0.9))
+        self.score_keys = score_keys
+        self.attn = None
+        if weighted:
+            g = torch.Generator(device=device)
+            g.manual_seed(seed + 7)
+            self.attn = torch.rand(us + (self.cap,), generator=g, device=device) * 0.9
 
     def head_tokens_per_step(self):
         return self.U * (self.N + self.B)
@@ -278,6 +286,10 @@ class Prefill:
             self.vd.vd_evict_block_holefill(self.cache, self.N, self.pos, pn, None, self.B,
                                             self.variant, self.mu, self.rs if self.mu else None,
                                             kept, scores)
+        elif self.score_keys or self.attn is not None:
+            self.vd.vd_evict_block_ex(self.cache, self.N, None, self.B, self.variant, self.mu,
+                                      self.rs if self.mu else None, self.score_keys, self.attn,
+                                      kept, scores)
         else:
             self.vd.vd_evict_block(self.cache, self.N, None, self.B, self.variant, self.mu,
                                    self.rs if self.mu else None, kept, scores)
@@ -312,9 +324,11 @@ class Prefill:
         rows read and written, running-sum state (and, hole-fill, the moved
         rows' positions)."""
         n, d = self.N + self.B, self.d
-        v_read = self.U * n * d * 2
+        v_read = self.U * n * d * 2          # the scored tensor (V, or K for the key-side rule)
         move = moved_rows_total * d * 2 * 2 * 2
         extra = self.U * d * 8 * 2 if self.mu else 0
+        if self.attn is not None:
+            extra += self.U * n * 4          # the attention weights
         if self.holefill:
             extra += moved_rows_total * 4 + self.U * self.B * 4
             return v_read + move + extra, v_read + self.U * self.B * d * 2 * 2 * 2 + extra
@@ -500,7 +514,8 @@ class Decode:
         return kk, vv, self.N + 1, self.N
 
 
-def make_workload(name, device, seed, mu, variant, n_seq=None, events=8, layout="ordered"):
+def make_workload(name, device, seed, mu, variant, n_seq=None, events=8, layout="ordered",
+                  **opts):
     """`events` = warm-up + timed steps: that many distinct blocks / tokens are
     pre-generated, up to the workload's own length (T / B blocks of the
     prompt, or its decode steps); longer runs reuse them in order."""
@@ -510,7 +525,7 @@ def make_workload(name, device, seed, mu, variant, n_seq=None, events=8, layout=
         cfg["n_seq"] = n_seq
     if cfg["kind"] == "prefill":
         pool = max(8, min(events, cfg["T"] // cfg["B"]))
-        return Prefill(name, cfg, device, seed, mu, variant, n_blocks=pool, layout=layout)
+        return Prefill(name, cfg, device, seed, mu, variant, n_blocks=pool, layout=layout, **opts)
     if cfg["kind"] == "decode":
         pool = max(8, min(events, cfg["steps"]))
         return Decode(name, cfg, device, seed, mu, variant, n_tokens=pool, layout=layout)
@@ -607,6 +622,41 @@ def measure_gpu(w, steps, warmup, device, e2e_steps):
                 bi=bi, bo=bo)
 
 
+def measure_dispersion(args, device, variant, peak, rank):
+    """vd_score_ex returning sigma_V per unit (Sec. 3.1) over the workload's
+    cache at steady state: one score-only launch per step; algorithmic bytes =
+    the V rows read once."""
+    import torch
+    import paper_2609_23314_gb300 as vd
+    from paper_2609_23314_gb300 import workloads as wl
+    _, cfg = wl.config(args.workload)
+    w = make_workload(args.workload, device, rank_seed(wl.BASE_SEED + cfg["index"], rank),
+                      vd.VD_MU_RECOMPUTE, vd.VD_SCORE_L2, args.n_seq, events=8)
+    sigma = torch.empty(w.cache.unit_shape(), device=device)
+    for _ in range(args.warmup):
+        vd.vd_score_ex(w.cache, vd.VD_SCORE_L2, False, None, sigma)
+    steps = args.extension_steps
+    start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    start.record()
+    for _ in range(steps):
+        vd.vd_score_ex(w.cache, vd.VD_SCORE_L2, False, None, sigma)
+    stop.record()
+    torch.cuda.synchronize()
+    ms = max_over_ranks(start.elapsed_time(stop), device) / steps
+    n = int(w.cache.len[0])
+    alg = w.U * n * w.d * 2 + w.U * 4
+    achieved = alg / (ms / 1e3) / 1e9
+    res = {"value": w.U * n / (ms / 1e3), "step_ms": ms,
+           "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                        "frac": achieved / peak, "kernel": "vd::evict_kernel<0, true, false> (score only)",
+                        "algorithmic_bytes_per_launch": alg, "kernel_ms": ms,
+                        "sigma_v_mean": float(sigma.mean().item())}}
+    del w
+    torch.cuda.empty_cache()
+    return res
+
+
 def cpu_baseline(w, budget_s=2.0, max_units=64):
     """The fp64 oracle (as it stands) on a bounded sample of the same events,
     on every host core; returns the extrapolated head-tokens/s."""
@@ -656,12 +706,13 @@ def run_vd(args):
     peak, peak_src = hbm_peak()
     from paper_2609_23314_gb300 import workloads as wl
 
-    def one(name, steps, layout="ordered"):
+    def one(name, steps, layout="ordered", mu_mode=None, **opts):
         _, cfg = wl.config(name)
         if args.n_seq:
             cfg["n_seq"] = args.n_seq
-        w = make_workload(name, device, rank_seed(wl.BASE_SEED + cfg["index"], rank), mu, variant,
-                          args.n_seq, events=args.warmup + steps, layout=layout)
+        w = make_workload(name, device, rank_seed(wl.BASE_SEED + cfg["index"], rank),
+                          mu if mu_mode is None else mu_mode, variant, args.n_seq,
+                          events=args.warmup + steps, layout=layout, **opts)
         m = measure_gpu(w, steps, args.warmup, device, min(steps, args.e2e_steps))
         step_ms = max_over_ranks(m["step_ms"], device) / steps
         kern_ms = max_over_ranks(m["kern_ms"], device)
@@ -714,6 +765,18 @@ def run_vd(args):
             r = one(name, args.holefill_steps, "holefill")
             release(r)
             holefill[name] = {k: r[k] for k in ("value", "step_ms", "roofline", "e2e")}
+    # scoring options on the primary (prefill) workload: the K-side rule (mean
+    # recomputed from K: K is read twice), attention weights, and the
+    # per-unit dispersion sigma_V from a score-only pass
+    extensions = {}
+    if args.extension_steps > 0 and wl.config(args.workload)[1]["kind"] == "prefill":
+        for key, opts, mu_mode in (("key_side", dict(score_keys=True), vd.VD_MU_RECOMPUTE),
+                                   ("attention_weighted", dict(weighted=True), None)):
+            r = one(args.workload, args.extension_steps, "ordered", mu_mode, **opts)
+            extensions[key] = {"value": r["value"], "step_ms": r["step_ms"],
+                               "roofline": r["roofline"]}
+            release(r)
+        extensions["dispersion"] = measure_dispersion(args, device, variant, peak, rank)
     if rank == 0:
         line = {
             "metric": METRIC, "value": primary["value"], "unit": UNIT, "n_gpus": ws,
@@ -735,6 +798,8 @@ def run_vd(args):
             line["secondary"]["clocks"] = secondary["m"]["clocks"]
         if holefill:
             line["holefill_layout"] = holefill
+        if extensions:
+            line["extensions"] = extensions
         print(json.dumps(line), flush=True)
     if ws > 1:
         import torch.distributed as dist
@@ -803,6 +868,8 @@ def main(argv=None):
     ap.add_argument("--secondary-steps", type=int, default=50)
     ap.add_argument("--layout", choices=["ordered", "holefill"], default="ordered",
                     help="cache layout of the primary and secondary measurements")
+    ap.add_argument("--extension-steps", type=int, default=50,
+                    help="steps of the key-side / weighted / dispersion measurements (0: skip)")
     ap.add_argument("--holefill-steps", type=int, default=50,
                     help="steps of the extra hole-fill-layout measurements (0: skip)")
     ap.add_argument("--mu", choices=["running", "recompute"], default="running")
