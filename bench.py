@@ -129,14 +129,14 @@ def kernel_source_hash() -> str:
     return h.hexdigest()[:16]
 
 
-def ncu_traffic(workload: str):
+def ncu_traffic(workload: str, layout: str = "ordered"):
     """DRAM bytes per launch of the eviction kernel from the committed ncu
     summary, if it was taken on the current kernel sources; else None."""
     path = os.path.join(ROOT, "profiles", "traffic.json")
     try:
         with open(path) as f:
             t = json.load(f)
-        e = t[workload]
+        e = t[workload if layout == "ordered" else f"{workload}:{layout}"]
         if e.get("source_hash") != kernel_source_hash():
             return None
         return float(e["dram_bytes_per_launch"])
@@ -726,7 +726,8 @@ def run_vd(args):
             "e2e": {"value": tok * ws / (e2e_ms / 1e3), "unit": UNIT,
                     "h2d_bytes_per_step": m["bi"], "d2h_bytes_per_step": m["bo"]},
             "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
-                         "frac": achieved / peak, "traffic": ncu_traffic(name),
+                         "frac": achieved / peak,
+                         "traffic": ncu_traffic(name, layout) if not opts else None,
                          "kernel": f"vd::evict_kernel<{variant}, {str(isinstance(w, Decode)).lower()}, "
                                    f"{str(layout == 'holefill').lower()}>",
                          "algorithmic_bytes_per_launch": alg,
