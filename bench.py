@@ -220,7 +220,7 @@ class Prefill:
     """Block boundary at steady state: append B rows, evict N + B -> N."""
 
     def __init__(self, name, cfg, device, seed, mu, variant, n_blocks=8, layout="ordered",
-                 score_keys=False, weighted=False):
+                 score_keys=False, weighted=False, dispersion=False):
         """n_blocks distinct appended blocks are pre-generated and reused in
         order; the benchmark asks for as many as the prompt has (T / B), so
         every timed event appends rows the cache has not seen.  layout
@@ -266,6 +266,8 @@ class Prefill:
             g = torch.Generator(device=device)
             g.manual_seed(seed + 7)
             self.attn = torch.rand(us + (self.cap,), generator=g, device=device) * 0.9
+        # per-unit sigma (Sec. 3.1) of the pre-eviction rows, from the score pass
+        self.sigma = torch.empty(us, device=device) if dispersion else None
 
     def head_tokens_per_step(self):
         return self.U * (self.N + self.B)
@@ -286,10 +288,10 @@ class Prefill:
             self.vd.vd_evict_block_holefill(self.cache, self.N, self.pos, pn, None, self.B,
                                             self.variant, self.mu, self.rs if self.mu else None,
                                             kept, scores)
-        elif self.score_keys or self.attn is not None:
+        elif self.score_keys or self.attn is not None or self.sigma is not None:
             self.vd.vd_evict_block_ex(self.cache, self.N, None, self.B, self.variant, self.mu,
                                       self.rs if self.mu else None, self.score_keys, self.attn,
-                                      kept, scores)
+                                      kept, scores, self.sigma)
         else:
             self.vd.vd_evict_block(self.cache, self.N, None, self.B, self.variant, self.mu,
                                    self.rs if self.mu else None, kept, scores)
@@ -622,6 +624,38 @@ def measure_gpu(w, steps, warmup, device, e2e_steps):
                 bi=bi, bo=bo)
 
 
+def graph_step_us(w, steps, device):
+    """Device time of one step (append + evict) with the host out of the
+    loop: `steps` steps captured once in a CUDA graph and replayed.  Small
+    workloads are otherwise bound by the host's launch rate."""
+    import torch
+    side = torch.cuda.Stream(device=device)
+    side.wait_stream(torch.cuda.current_stream(device))
+    with torch.cuda.stream(side):
+        for _ in range(3):
+            w.step()
+    torch.cuda.current_stream(device).wait_stream(side)
+    torch.cuda.synchronize(device)
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        for _ in range(steps):
+            w.step()
+    for _ in range(3):
+        g.replay()
+    start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    reps = 20
+    torch.cuda.synchronize(device)
+    start.record()
+    for _ in range(reps):
+        g.replay()
+    stop.record()
+    torch.cuda.synchronize(device)
+    status = w.vd.vd_get_device_status()
+    if status != 0:
+        raise RuntimeError(f"device status {status}: {w.vd.vd_status_string(status)}")
+    return start.elapsed_time(stop) * 1e3 / (reps * steps)
+
+
 def measure_dispersion(args, device, variant, peak, rank):
     """vd_score_ex returning sigma_V per unit (Sec. 3.1) over the workload's
     cache at steady state: one score-only launch per step; algorithmic bytes =
@@ -644,6 +678,10 @@ def measure_dispersion(args, device, variant, peak, rank):
     stop.record()
     torch.cuda.synchronize()
     ms = max_over_ranks(start.elapsed_time(stop), device) / steps
+    # the realized sigma_V / sigma_K of the generator (untimed)
+    sigma_k = torch.empty_like(sigma)
+    vd.vd_score_ex(w.cache, vd.VD_SCORE_L2, True, None, sigma_k)
+    ratio = float((sigma / sigma_k).mean().item())
     n = int(w.cache.len[0])
     alg = w.U * n * w.d * 2 + w.U * 4
     achieved = alg / (ms / 1e3) / 1e9
@@ -651,7 +689,9 @@ def measure_dispersion(args, device, variant, peak, rank):
            "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                         "frac": achieved / peak, "kernel": "vd::evict_kernel<0, true, false> (score only)",
                         "algorithmic_bytes_per_launch": alg, "kernel_ms": ms,
-                        "sigma_v_mean": float(sigma.mean().item())}}
+                        "sigma_v_mean": float(sigma.mean().item()),
+                        "sigma_k_mean": float(sigma_k.mean().item()),
+                        "sigma_v_over_sigma_k": ratio}}
     del w
     torch.cuda.empty_cache()
     return res
@@ -679,9 +719,32 @@ def cpu_baseline(w, budget_s=2.0, max_units=64):
         elapsed += time.perf_counter() - t0
         events += 1
     rate = units * n * events / elapsed
+    # one thread on a smaller sample of the same units
+    u1 = min(units, 4)
+    k, v = k0[:u1].copy(), v0[:u1].copy()
+    t0 = time.perf_counter()
+    orc.evict_units(k, v, lens[:u1], Ns[:u1], 1, var, nthreads=1)
+    rate1 = u1 * n / (time.perf_counter() - t0)
     return {"value": rate, "unit": UNIT, "cores": cores, "kind": "oracle",
+            "single_thread_value": rate1, "cpu_model": cpu_model(),
             "sample": f"{units} of {w.U} units x {events} events of {w.name} at n={n} -> N={N}; "
-                      f"fp64 C oracle, one POSIX thread per core, {elapsed:.2f} s wall"}
+                      f"fp64 C oracle, one POSIX thread per core, {elapsed:.2f} s wall; "
+                      f"single thread: {u1} units x 1 event"}
+
+
+def cpu_model():
+    """The host CPU's model name (x86 'model name', or the Arm part and
+    implementer from /proc/cpuinfo)."""
+    try:
+        with open("/proc/cpuinfo") as f:
+            info = f.read()
+    except OSError:
+        return "unknown"
+    for key in ("model name", "Model", "CPU part"):
+        for line in info.splitlines():
+            if line.startswith(key) and ":" in line:
+                return line.split(":", 1)[1].strip()
+    return "unknown"
 
 
 def run_vd(args):
@@ -757,6 +820,16 @@ def run_vd(args):
     if args.secondary not in ("", "none") and args.secondary != args.workload:
         secondary = one(args.secondary, args.secondary_steps, args.layout)
         release(secondary)
+    # the smallest workload's per-event latency (a few units: launch- and
+    # latency-bound, reported in microseconds)
+    latency = None
+    if args.latency_steps > 0:
+        r = one("tiny_prefill", args.latency_steps)
+        latency = {"workload": "tiny_prefill", "event_us": r["step_ms"] * 1e3,
+                   "kernel_us": r["kern_ms"] * 1e3, "e2e_event_us":
+                   r["w"].head_tokens_per_step() * ws / r["e2e"]["value"] * 1e6,
+                   "graph_event_us": graph_step_us(r["w"], args.latency_steps, device)}
+        release(r)
     # the hole-fill cache layout (a next row: same policy, fewest rows moved)
     holefill = {}
     if args.holefill_steps > 0 and args.layout == "ordered":
@@ -768,14 +841,18 @@ def run_vd(args):
             holefill[name] = {k: r[k] for k in ("value", "step_ms", "roofline", "e2e")}
     # scoring options on the primary (prefill) workload: the K-side rule (mean
     # recomputed from K: K is read twice), attention weights, and the
-    # per-unit dispersion sigma_V from a score-only pass
+    # per-unit dispersion sigma_V from a score-only pass, and as a by-product
+    # of the eviction's own score pass
     extensions = {}
     if args.extension_steps > 0 and wl.config(args.workload)[1]["kind"] == "prefill":
         for key, opts, mu_mode in (("key_side", dict(score_keys=True), vd.VD_MU_RECOMPUTE),
-                                   ("attention_weighted", dict(weighted=True), None)):
+                                   ("attention_weighted", dict(weighted=True), None),
+                                   ("dispersion_by_product", dict(dispersion=True), None)):
             r = one(args.workload, args.extension_steps, "ordered", mu_mode, **opts)
             extensions[key] = {"value": r["value"], "step_ms": r["step_ms"],
                                "roofline": r["roofline"]}
+            if r["w"].sigma is not None:
+                extensions[key]["sigma_v_mean"] = float(r["w"].sigma.mean().item())
             release(r)
         extensions["dispersion"] = measure_dispersion(args, device, variant, peak, rank)
     if rank == 0:
@@ -797,6 +874,8 @@ def run_vd(args):
             line["secondary"] = {k: secondary[k] for k in ("workload", "value", "step_ms", "roofline",
                                                            "e2e", "config")}
             line["secondary"]["clocks"] = secondary["m"]["clocks"]
+        if latency is not None:
+            line["latency"] = latency
         if holefill:
             line["holefill_layout"] = holefill
         if extensions:
@@ -876,6 +955,8 @@ def main(argv=None):
     ap.add_argument("--mu", choices=["running", "recompute"], default="running")
     ap.add_argument("--variant", choices=["l2", "dir", "norm"], default="l2")
     ap.add_argument("--e2e-steps", type=int, default=50)
+    ap.add_argument("--latency-steps", type=int, default=12,
+                    help="events of the tiny_prefill latency measurement (0: skip)")
     ap.add_argument("--n-seq", type=int, default=None,
                     help="override the workload's number of sequences (smaller profiling cases)")
     ap.add_argument("--no-cpu-baseline", action="store_true")

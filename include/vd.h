@@ -63,7 +63,9 @@ typedef enum {
                              on append, or B > len in running-sum mode */
   VD_ERR_DEVICE_BUDGET = 8, /* device: N_dev[s] out of [1, N], or a decode call found
                                len > N + 1 */
-  VD_ERR_NO_DEVICE = 9    /* no CUDA device, or not an sm_103 device */
+  VD_ERR_NO_DEVICE = 9,   /* no CUDA device, or not an sm_103 device */
+  VD_ERR_INTERNAL = 10    /* device: a kernel's self-check found an inconsistent slot
+                             list (never expected); the access was skipped */
 } vd_status;
 
 /* Scoring rules of Sec. 3.2.  Higher scores are kept.
@@ -159,12 +161,18 @@ vd_status vd_score_ex(const vd_cache* c, vd_variant var, int32_t score_keys, flo
  *               Eq. (app_fastcaote) (with VD_SCORE_L2).  A weight outside
  *               [0, 1) gives a NaN score (ranked lowest, VD_ERR_NONFINITE).
  *               scores_out then holds the weighted scores.
+ *   dispersion_out  nullable fp32 device [n_seq][n_layer][n_kv_head]: sigma of
+ *               Sec. 3.1 over the len pre-eviction rows (sigma_V, or sigma_K
+ *               with score_keys), from the same score pass (no extra read);
+ *               the unweighted L2 distances; requires var == VD_SCORE_L2
+ *               (else VD_ERR_INVALID_ARG).  Written only for units that
+ *               evicted, like scores_out.
  * Other arguments as in vd_evict_block.  A weighted decode step is this call
  * with B = 1. */
 vd_status vd_evict_block_ex(const vd_cache* c, int32_t N, const int32_t* N_dev, int32_t B,
                             vd_variant var, vd_mu_mode mu, double* running_sum,
                             int32_t score_keys, const float* attn, int32_t* kept_idx_out,
-                            float* scores_out, vd_stream_t stream);
+                            float* scores_out, float* dispersion_out, vd_stream_t stream);
 
 /* Hole-fill layout (not in the paper; its eviction rule with a cache layout
  * that moves as few rows as possible).  Same policy as vd_evict_block /

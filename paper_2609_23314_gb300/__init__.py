@@ -71,7 +71,7 @@ def load_library() -> ctypes.CDLL:
             lib.vd_evict_block_holefill.argtypes = [cp, I32, P, I32, S, S, P, P, P, P, P, P]
             lib.vd_evict_decode_holefill.argtypes = [cp, I32, P, S, S, P, P, P, P, P, P, P]
             lib.vd_score_ex.argtypes = [cp, S, I32, P, P, P]
-            lib.vd_evict_block_ex.argtypes = [cp, I32, P, I32, S, S, P, I32, P, P, P, P]
+            lib.vd_evict_block_ex.argtypes = [cp, I32, P, I32, S, S, P, I32, P, P, P, P, P]
             lib.vd_append.argtypes = [cp, P, P, I32, P]
             lib.vd_running_sum_init.argtypes = [cp, P, P]
             lib.vd_workspace_size.argtypes = [cp]
@@ -218,8 +218,11 @@ def vd_score_ex(cache: Cache, variant: int, score_keys: bool = False, scores_out
 
 def vd_evict_block_ex(cache: Cache, N: int, N_dev=None, B: int = 0, variant: int = VD_SCORE_L2,
                       mu: int = VD_MU_RECOMPUTE, running_sum=None, score_keys: bool = False,
-                      attn=None, kept_idx_out=None, scores_out=None, stream=None) -> None:
-    """Block eviction on the K-side rule and/or with attention weights."""
+                      attn=None, kept_idx_out=None, scores_out=None, dispersion_out=None,
+                      stream=None) -> None:
+    """Block eviction on the K-side rule and/or with attention weights;
+    dispersion_out: fp32 [n_seq, n_layer, n_kv_head], sigma of the
+    pre-eviction rows from the same score pass (units that evicted)."""
     torch = _torch()
     us = cache.unit_shape()
     args = (
@@ -228,10 +231,11 @@ def vd_evict_block_ex(cache: Cache, N: int, N_dev=None, B: int = 0, variant: int
         _ptr(attn, torch.float32, us + (cache.capacity,), "attn", cache.device),
         _ptr(kept_idx_out, torch.int32, us + (int(N),), "kept_idx_out", cache.device),
         _ptr(scores_out, torch.float32, us + (cache.capacity,), "scores_out", cache.device),
+        _ptr(dispersion_out, torch.float32, us, "dispersion_out", cache.device),
     )
     _check(load_library().vd_evict_block_ex(cache.ref(), int(N), args[0], int(B), int(variant),
                                             int(mu), args[1], int(bool(score_keys)), args[2],
-                                            args[3], args[4], _stream(stream)),
+                                            args[3], args[4], args[5], _stream(stream)),
            "vd_evict_block_ex")
 
 

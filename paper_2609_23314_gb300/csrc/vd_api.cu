@@ -100,11 +100,23 @@ __global__ void __launch_bounds__(kThreads) vd_rsum_init_kernel(const uint16_t* 
 // ---------------------------------------------------------------------------
 namespace {
 
+// A cluster-size decision for one launch shape (the occupancy queries behind
+// it cost more host time than a small eviction takes on the device).
+struct ClusterChoice {
+  const void* kern;
+  long long units;
+  int d, capacity, with_select, want, c;
+  size_t smem;
+};
+constexpr int kChoiceSlots = 32;
+
 struct DeviceState {
   bool ready = false;
   unsigned* status = nullptr;
   int sms = 0;
   int smem_optin = 0;
+  ClusterChoice choice[kChoiceSlots];  // guarded by g_mu; replaced round-robin
+  int n_choice = 0, next_choice = 0;
 };
 
 constexpr int kMaxDevices = 64;
@@ -209,12 +221,10 @@ bool cluster_allowed(int c, int d) {
 // least two waves, so that no short tail wave runs alone; with none such,
 // the largest allowed C.  (Measured on GB300: a 1.1-wave launch loses ~15%,
 // while larger clusters than needed pay for extra synchronisation and
-// narrower row segments.)  VD_CLUSTER_SIZE (1, 2, 4, 8 or 16) overrides the
-// choice, for tuning.
+// narrower row segments.)  want (VD_CLUSTER_SIZE: 1, 2, 4, 8 or 16)
+// overrides the choice, for tuning.
 int choose_cluster(const void* kern, long long units, int d, int capacity, bool with_select,
-                   const DeviceState& st, size_t* smem_out) {
-  const char* env = std::getenv("VD_CLUSTER_SIZE");
-  const int want = env ? std::atoi(env) : 0;
+                   int want, const DeviceState& st, size_t* smem_out) {
   int chosen = 0, largest = 1;
   for (int c = 1; c <= 16; c *= 2) {
     if (want >= 1 && c != want) continue;
@@ -238,6 +248,31 @@ int choose_cluster(const void* kern, long long units, int d, int capacity, bool 
   if (chosen == 0) chosen = largest;
   *smem_out = vd::smem_layout(capacity, chosen, with_select).total;
   return chosen;
+}
+
+// choose_cluster, remembered per launch shape.
+int cached_cluster(const void* kern, long long units, int d, int capacity, bool with_select,
+                   DeviceState& st, size_t* smem_out) {
+  const char* env = std::getenv("VD_CLUSTER_SIZE");
+  const int want = env ? std::atoi(env) : 0;
+  const int ws = with_select ? 1 : 0;
+  {
+    std::lock_guard<std::mutex> lk(g_mu);
+    for (int i = 0; i < st.n_choice; ++i) {
+      const ClusterChoice& e = st.choice[i];
+      if (e.kern == kern && e.units == units && e.d == d && e.capacity == capacity &&
+          e.with_select == ws && e.want == want) {
+        *smem_out = e.smem;
+        return e.c;
+      }
+    }
+  }
+  const int c = choose_cluster(kern, units, d, capacity, with_select, want, st, smem_out);
+  std::lock_guard<std::mutex> lk(g_mu);
+  st.choice[st.next_choice] = ClusterChoice{kern, units, d, capacity, ws, want, c, *smem_out};
+  st.next_choice = (st.next_choice + 1) % kChoiceSlots;
+  if (st.n_choice < kChoiceSlots) ++st.n_choice;
+  return c;
 }
 
 vd_status launch(const void* kern, long long units, int c, size_t smem, const vd::EvictArgs& a,
@@ -278,7 +313,7 @@ vd_status run(const vd_cache* c, int32_t N, const int32_t* N_dev, int32_t B, vd_
   } else if (!scores_out && !disp_out) {
     return VD_ERR_INVALID_ARG;
   }
-  if (disp_out && (!score_only || var != VD_SCORE_L2)) return VD_ERR_INVALID_ARG;
+  if (disp_out && (decode || var != VD_SCORE_L2)) return VD_ERR_INVALID_ARG;
   if (weights && (score_only || decode)) return VD_ERR_INVALID_ARG;
   if (score_k && mu == VD_MU_RUNNING && !score_only) return VD_ERR_UNSUPPORTED;
   const bool holefill = pos != nullptr || pos_new != nullptr;
@@ -320,7 +355,7 @@ vd_status run(const vd_cache* c, int32_t N, const int32_t* N_dev, int32_t B, vd_
   a.weights = weights;
   a.disp_out = disp_out;
   size_t smem = 0;
-  a.cluster = choose_cluster(kern, units, c->head_dim, c->capacity, !small, *st, &smem);
+  a.cluster = cached_cluster(kern, units, c->head_dim, c->capacity, !small, *st, &smem);
   if (smem > (size_t)st->smem_optin) return VD_ERR_UNSUPPORTED;
 
   r = launch(kern, units, a.cluster, smem, a, s);
@@ -368,10 +403,10 @@ vd_status vd_score_ex(const vd_cache* c, vd_variant var, int32_t score_keys, flo
 vd_status vd_evict_block_ex(const vd_cache* c, int32_t N, const int32_t* N_dev, int32_t B,
                             vd_variant var, vd_mu_mode mu, double* running_sum,
                             int32_t score_keys, const float* attn, int32_t* kept_idx_out,
-                            float* scores_out, vd_stream_t stream) {
+                            float* scores_out, float* dispersion_out, vd_stream_t stream) {
   return run(c, N, N_dev, B, var, mu, running_sum, nullptr, kept_idx_out, scores_out,
              reinterpret_cast<cudaStream_t>(stream), false, false, nullptr, nullptr, score_keys,
-             attn, nullptr);
+             attn, dispersion_out);
 }
 
 vd_status vd_evict_block_holefill(const vd_cache* c, int32_t N, const int32_t* N_dev, int32_t B,
@@ -451,6 +486,7 @@ const char* vd_status_string(vd_status st) {
     case VD_ERR_DEVICE_LEN: return "device: sequence length out of range";
     case VD_ERR_DEVICE_BUDGET: return "device: budget out of range or decode over budget";
     case VD_ERR_NO_DEVICE: return "no sm_103 CUDA device";
+    case VD_ERR_INTERNAL: return "device: inconsistent slot list (internal self-check)";
     default: return "unknown status";
   }
 }

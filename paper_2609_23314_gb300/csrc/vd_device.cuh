@@ -18,6 +18,7 @@ constexpr unsigned kFull = 0xffffffffu;
 constexpr unsigned kStNonfinite = 4;
 constexpr unsigned kStDeviceLen = 7;
 constexpr unsigned kStDeviceBudget = 8;
+constexpr unsigned kStInternal = 10;
 
 // First anomaly wins; later ones are dropped.  Never traps.
 __device__ __forceinline__ void record_status(unsigned* st, unsigned code) {

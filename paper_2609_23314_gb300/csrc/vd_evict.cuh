@@ -94,7 +94,7 @@ struct EvictArgs {
   int32_t holefill;        // 1: hole-fill layout (ties by position), 0: ordered
   int32_t score_k;         // 1: mean and scores from K (key-side rules)
   const float* weights;    // nullable [U][capacity]: attention weights a_j (block path)
-  float* disp_out;         // nullable [U]: std of the L2 scores (score-only path)
+  float* disp_out;         // nullable [U]: std of the L2 scores of the scored rows
 };
 
 // Fixed part of the dynamic shared memory.  After it (16-byte aligned): the
@@ -252,6 +252,59 @@ __device__ __forceinline__ uint32_t score_key(float s, bool& bad) {
   return (s == s) ? __float_as_uint(s) : 0u;
 }
 
+// Dispersion of the L2 scores over a unit (Sec. 3.1: sigma = std_j s_j):
+// every thread's double-float sums of s and s^2 are merged in a fixed order
+// into this CTA's S.disp (ends with a block barrier).  wsc: 4 * kWarps floats
+// of block-private scratch (peer CTAs may still be reading S.acc_*).
+__device__ __forceinline__ void disp_reduce_cta(float ds_hi, float ds_lo, float dq_hi,
+                                                float dq_lo, float* wsc, Smem& S) {
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  ff a1 = ff_add(ff{ds_hi, 0.f}, ff{0.f, ds_lo});
+  ff a2 = ff_add(ff{dq_hi, 0.f}, ff{0.f, dq_lo});
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+    a1 = ff_add(a1, ff_shfl_xor(a1, off));
+    a2 = ff_add(a2, ff_shfl_xor(a2, off));
+  }
+  if (lane == 0) {
+    wsc[warp] = a1.hi;
+    wsc[kWarps + warp] = a1.lo;
+    wsc[2 * kWarps + warp] = a2.hi;
+    wsc[3 * kWarps + warp] = a2.lo;
+  }
+  __syncthreads();
+  if (tid == 0) {
+    ff t1{0.f, 0.f}, t2{0.f, 0.f};
+    for (int w = 0; w < kWarps; ++w) {
+      t1 = ff_add(t1, ff{wsc[w], wsc[kWarps + w]});
+      t2 = ff_add(t2, ff{wsc[2 * kWarps + w], wsc[3 * kWarps + w]});
+    }
+    S.disp[0] = t1.hi;
+    S.disp[1] = t1.lo;
+    S.disp[2] = t2.hi;
+    S.disp[3] = t2.lo;
+  }
+  __syncthreads();
+}
+
+// sigma = sqrt(E[s^2] - E[s]^2) from the S.disp of the cluster's C CTAs, in
+// rank order (one thread; every CTA's S.disp must be complete and its CTA
+// still resident).
+__device__ __forceinline__ float disp_finish(Smem& S, int C, int n) {
+  double s1 = 0.0, s2 = 0.0;
+  const uint32_t base = smem_addr(&S.disp[0]);
+  for (int rr = 0; rr < C; ++rr) {
+    float v[4];
+    for (int k = 0; k < 4; ++k)
+      v[k] = C > 1 ? ld_cluster_f32(mapa(base + 4u * (unsigned)k, (unsigned)rr)) : S.disp[k];
+    s1 += (double)v[0] + (double)v[1];
+    s2 += (double)v[2] + (double)v[3];
+  }
+  const double m = s1 / (double)n;
+  const double var = s2 / (double)n - m * m;
+  return (float)sqrt(var > 0.0 ? var : 0.0);
+}
+
 // Radix select over the keys of the whole cluster: t = the N-th largest key
 // (1-based), keep_eq = how many keys equal to t survive, cnt_eq = how many
 // keys equal t.  key_of(j, ok) gives the key of this CTA's j-th row (j < R)
@@ -340,12 +393,14 @@ __device__ __forceinline__ Selection cluster_radix_select(KeyOf key_of, int R, i
 // into perm[] of every CTA of the cluster: kept slots ascending at [0, N),
 // evicted slots ascending at [N, n).  Threads own contiguous row chunks, so
 // prefix sums follow slot order (ties go to the lower slot).  Ends with the
-// cluster barrier after which every CTA's perm[] is complete.
+// cluster barrier after which every CTA's perm[] is complete.  A position
+// outside [0, n) (impossible for a consistent selection) is skipped and
+// recorded as kStInternal.
 template <bool by_tiekey, class TieKey>
 __device__ __forceinline__ void cluster_build_perm(const uint32_t* keys, int r0, int R, int N,
-                                                   Selection sel, uint32_t t2, TieKey tiekey,
-                                                   int C, unsigned rank, uint16_t* perm,
-                                                   Smem& S) {
+                                                   int n, Selection sel, uint32_t t2,
+                                                   TieKey tiekey, int C, unsigned rank,
+                                                   uint16_t* perm, unsigned* status, Smem& S) {
   const int tid = threadIdx.x;
   const int ch = (R + kThreads - 1) / kThreads;
   const int c0 = min(R, tid * ch), c1 = min(R, c0 + ch);
@@ -387,6 +442,10 @@ __device__ __forceinline__ void cluster_build_perm(const uint32_t* keys, int r0,
     const int row = r0 + j;
     const int pos = keep ? kp : N + (row - kp);
     kp += keep;
+    if ((unsigned)pos >= (unsigned)n) {  // self-check: a consistent selection never gets here
+      record_status(status, kStInternal);
+      continue;
+    }
     if (C > 1) {
       for (int cc = 0; cc < C; ++cc)
         st_cluster_u16(mapa(perm_addr + 2u * (unsigned)pos, (unsigned)cc), (uint16_t)row);
@@ -399,10 +458,13 @@ __device__ __forceinline__ void cluster_build_perm(const uint32_t* keys, int r0,
 
 // In-place, order-preserving move of rows [r_begin, r_end) of the column
 // slice [chunk0, chunk0 + cps) of the concatenated [K | V] row: row r takes
-// source row perm[r] (or r + 1 when perm is null: the decode shift).
+// source row perm[r] (or r + 1 when perm is null: the decode shift).  A
+// source at or above n (impossible for a consistent slot list) is not read
+// and is recorded as kStInternal (its row then holds unspecified bytes).
 __device__ __forceinline__ void compact_slice(uint16_t* kb, uint16_t* vb, int d, int chunk0,
-                                              int cps, int r_begin, int r_end,
-                                              const uint16_t* perm, uint32_t ring) {
+                                              int cps, int r_begin, int r_end, int n,
+                                              const uint16_t* perm, unsigned* status,
+                                              uint32_t ring) {
   const int tid = threadIdx.x;
   const int d8 = d >> 3;
   const int rs = kThreads / cps;
@@ -423,7 +485,10 @@ __device__ __forceinline__ void compact_slice(uint16_t* kb, uint16_t* vb, int d,
         const int r = r_begin + t * tile + u * rs + my_off;
         if (on && r < r_end) {
           const int src = perm ? (int)perm[r] : r + 1;
-          cp_async16(slot(t % kRingStages, u), col + (size_t)src * d);
+          if (src < n)
+            cp_async16(slot(t % kRingStages, u), col + (size_t)src * d);
+          else
+            record_status(status, kStInternal);
         }
       }
     }
@@ -445,10 +510,13 @@ __device__ __forceinline__ void compact_slice(uint16_t* kb, uint16_t* vb, int d,
 
 // Hole-fill layout: move h rows, row src_of(i) -> row dst_of(i), of the
 // column slice [chunk0, chunk0 + cps) of [K | V].  Every source lies at or
-// above N and every destination below it, so the moves are independent.
+// above N and every destination below it, so the moves are independent.  A
+// row outside [0, n) (impossible for a consistent slot list) is skipped and
+// recorded as kStInternal.
 template <class SrcOf, class DstOf>
 __device__ __forceinline__ void move_rows(uint16_t* kb, uint16_t* vb, int d, int chunk0, int cps,
-                                          int h, SrcOf src_of, DstOf dst_of) {
+                                          int h, int n, SrcOf src_of, DstOf dst_of,
+                                          unsigned* status) {
   const int d8 = d >> 3;
   const int items = h * cps;
   constexpr int U = 4;
@@ -462,8 +530,13 @@ __device__ __forceinline__ void move_rows(uint16_t* kb, uint16_t* vb, int d, int
       if (it < items) {
         const int i = it / cps, c = chunk0 + it % cps;
         uint16_t* col = c < d8 ? kb + c * 8 : vb + (c - d8) * 8;
-        q[k] = ld_cg16(col + (size_t)src_of(i) * d);
-        dstp[k] = col + (size_t)dst_of(i) * d;
+        const int sr = src_of(i), dr = dst_of(i);
+        if ((unsigned)sr < (unsigned)n && (unsigned)dr < (unsigned)n) {
+          q[k] = ld_cg16(col + (size_t)sr * d);
+          dstp[k] = col + (size_t)dr * d;
+        } else {
+          record_status(status, kStInternal);
+        }
       }
     }
 #pragma unroll
@@ -602,6 +675,8 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
   if (score_split) cluster_arrive();
 
   // ---- 2. scores -------------------------------------------------------
+  // sigma of the L2 scores (host-checked; compiled into the L2 kernels only)
+  const bool disp = VAR == 0 && a.disp_out != nullptr;
   {
     const int ci = lane & (lpr - 1);
     const bool active = ci < d8;
@@ -613,7 +688,6 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
     }
     const bool mu_zero = VAR == 1 && S.mu_zero;
     const bool weighted = !DECODE && a.weights != nullptr;
-    const bool disp = a.score_only && a.disp_out != nullptr;
     float ds_hi = 0.f, ds_lo = 0.f, dq_hi = 0.f, dq_lo = 0.f;  // dispersion sums
     unsigned long long best = ~0ull;  // (key, tie-break) of this thread's minimum
     unsigned best_key = 0xffffffffu;   // hole-fill: key of this thread's minimum
@@ -658,7 +732,7 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
           if (in && ci == 0) {
             const int r = r0 + item;
             if (sc_out && !weighted) sc_out[r] = s;
-            if (disp) {  // sum s and s^2 (the square split exactly by an FMA)
+            if (VAR == 0 && disp) {  // sum s and s^2 (the square split exactly by an FMA)
               ff_accumulate(ds_hi, ds_lo, s);
               const float q2 = s * s;
               ff_accumulate(dq_hi, dq_lo, q2);
@@ -688,53 +762,19 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
           }
         },
         ring);
+    // sigma is defined on the L2 distance (VAR 0), whose scores never read
+    // muhat: it serves as the scratch
+    if constexpr (VAR == 0) {
+      if (disp) disp_reduce_cta(ds_hi, ds_lo, dq_hi, dq_lo, S.muhat, S);
+    }
     if (a.score_only) {
       if (score_split) cluster_wait();
-      if (disp) {
-        // dispersion of the scores over the unit: std_j s_j = sqrt(E[s^2] - E[s]^2),
-        // the CTA sums merged in a fixed order, then across the cluster
-        ff a1 = ff_add(ff{ds_hi, 0.f}, ff{0.f, ds_lo});
-        ff a2 = ff_add(ff{dq_hi, 0.f}, ff{0.f, dq_lo});
-#pragma unroll
-        for (int off = 16; off > 0; off >>= 1) {
-          a1 = ff_add(a1, ff_shfl_xor(a1, off));
-          a2 = ff_add(a2, ff_shfl_xor(a2, off));
+      if constexpr (VAR == 0) {
+        if (disp) {
+          if (C > 1) cluster_sync();
+          if (rank == 0 && tid == 0) a.disp_out[u] = disp_finish(S, C, n);
+          if (C > 1) cluster_sync();  // peers stay until rank 0 has read them
         }
-        if (lane == 0) {
-          S.acc_hi[warp] = a1.hi;
-          S.acc_lo[warp] = a1.lo;
-          S.acc_hi[32 + warp] = a2.hi;
-          S.acc_lo[32 + warp] = a2.lo;
-        }
-        __syncthreads();
-        if (tid == 0) {
-          ff t1{0.f, 0.f}, t2{0.f, 0.f};
-          for (int w = 0; w < kWarps; ++w) {
-            t1 = ff_add(t1, ff{S.acc_hi[w], S.acc_lo[w]});
-            t2 = ff_add(t2, ff{S.acc_hi[32 + w], S.acc_lo[32 + w]});
-          }
-          S.disp[0] = t1.hi;
-          S.disp[1] = t1.lo;
-          S.disp[2] = t2.hi;
-          S.disp[3] = t2.lo;
-        }
-        if (C > 1) cluster_sync(); else __syncthreads();
-        if (rank == 0 && tid == 0) {
-          double s1 = 0.0, s2 = 0.0;
-          for (int rr = 0; rr < C; ++rr) {
-            const uint32_t base = smem_addr(&S.disp[0]);
-            float v[4];
-            for (int k = 0; k < 4; ++k)
-              v[k] = C > 1 ? ld_cluster_f32(mapa(base + 4u * (unsigned)k, (unsigned)rr))
-                           : S.disp[k];
-            s1 += (double)v[0] + (double)v[1];
-            s2 += (double)v[2] + (double)v[3];
-          }
-          const double m = s1 / (double)n;
-          const double var = s2 / (double)n - m * m;
-          a.disp_out[u] = (float)sqrt(var > 0.0 ? var : 0.0);
-        }
-        if (C > 1) cluster_sync();  // peers stay until rank 0 has read them
       }
       return;
     }
@@ -816,6 +856,9 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
           return keys[j];
         },
         R, Nb, C, S);
+    if constexpr (VAR == 0) {
+      if (disp && rank == 0 && tid == 0) a.disp_out[u] = disp_finish(S, C, n);
+    }
     // hole-fill layout: the surviving ties are the lowest positions, found
     // by a second select over the complemented positions of the tied rows
     uint32_t t2 = 0u;
@@ -828,8 +871,9 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
           R, sel.keep_eq, C, S);
       t2 = s2.t;
     }
-    cluster_build_perm<HF>(keys, r0, R, Nb, sel, t2,
-                           [&](int j) { return ~(uint32_t)pos_of(r0 + j); }, C, rank, perm, S);
+    cluster_build_perm<HF>(keys, r0, R, Nb, n, sel, t2,
+                           [&](int j) { return ~(uint32_t)pos_of(r0 + j); }, C, rank, perm,
+                           a.status, S);
     e_first = perm[Nb];
   }
 
@@ -851,7 +895,11 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
     const int B = VAR != 2 ? 0 : a.B;
     sum_rows(vb, d, vchunk0, vchunks, vp, B + (n - Nb),
              [&](int i) {
-               return i < B ? first_new + i : (DECODE ? e_first : (int)perm[Nb + (i - B)]);
+               const int r =
+                   i < B ? first_new + i : (DECODE ? e_first : (int)perm[Nb + (i - B)]);
+               if ((unsigned)r < (unsigned)n) return r;
+               record_status(a.status, kStInternal);  // self-check: never expected
+               return 0;
              },
              [&](int i) { return i < B ? 1.f : -1.f; }, S, ring);
     if (tid < vchunks * 8) {
@@ -864,7 +912,8 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
 
   // ---- 6. in-place compaction of this CTA's column slice ---------------
   if constexpr (!HF) {
-    compact_slice(kb, vb, d, chunk0, cps, e_first, Nb, DECODE ? nullptr : perm, ring);
+    compact_slice(kb, vb, d, chunk0, cps, e_first, Nb, n, DECODE ? nullptr : perm, a.status,
+                  ring);
   } else {
     // hole-fill: the kept rows at or above N move into the evicted slots
     // below N, in ascending order (movers: the tail of the kept list; holes:
@@ -886,7 +935,7 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
     }
     auto src = [&](int i) { return DECODE ? n - 1 : (int)perm[Nb - h + i]; };
     auto dst = [&](int i) { return DECODE ? e_first : (int)perm[Nb + i]; };
-    move_rows(kb, vb, d, chunk0, cps, h, src, dst);
+    move_rows(kb, vb, d, chunk0, cps, h, n, src, dst, a.status);
     if (rank == 0) {
       for (int r = max(first_new, 0) + tid; r < Nb; r += kThreads) posu[r] = pnew + (r - first_new);
       int32_t* ko = a.kept_out ? a.kept_out + (size_t)u * a.N : nullptr;
@@ -895,6 +944,7 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
       __syncthreads();
       for (int i = tid; i < h; i += kThreads) {
         const int sr = src(i), dr = dst(i);
+        if ((unsigned)sr >= (unsigned)n || (unsigned)dr >= (unsigned)n) continue;  // recorded
         posu[dr] = pos_of(sr);
         if (ko) ko[dr] = sr;
       }

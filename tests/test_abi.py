@@ -84,3 +84,22 @@ def test_bad_arguments_rejected_before_launch(lib):
     assert lib.vd_append(ref, None, None, 4, None) == 1
     assert lib.vd_append(ref, 0x18, 0x28, 4, None) == 2                               # unaligned rows
     assert lib.vd_running_sum_init(ref, None, None) == 1
+
+
+def test_scoring_options_rejected_before_launch(lib):
+    c = _cache()
+    ref = ctypes.byref(c)
+    sigma = 0x40
+    # sigma is defined on the L2 distance
+    assert lib.vd_evict_block_ex(ref, 16, None, 4, 1, 0, None, 0, None, None, None, sigma,
+                                 None) == 1
+    assert lib.vd_score_ex(ref, 2, 0, None, sigma, None) == 1
+    assert lib.vd_score_ex(ref, 0, 0, None, None, None) == 1                  # no output
+    # the running sum tracks V: the K-side rule recomputes its mean
+    assert lib.vd_evict_block_ex(ref, 16, None, 4, 0, 1, 0x80, 1, None, None, None, None,
+                                 None) == 3
+    # the hole-fill layout needs both position arrays
+    assert lib.vd_evict_block_holefill(ref, 16, None, 4, 0, 0, None, 0x40, None, None, None,
+                                       None) == 1
+    assert lib.vd_evict_decode_holefill(ref, 16, None, 0, 0, None, None, 0x40, None, None,
+                                        None, None) == 1

@@ -144,6 +144,62 @@ def test_dispersion_matches_oracle(orc, keys, cluster, monkeypatch):
         assert abs(got[u] - want) <= 1e-5 * want + 1e-6, (u, got[u], want)
 
 
+@pytest.mark.parametrize("keys", [False, True], ids=["sigma_v", "sigma_k"])
+@pytest.mark.parametrize("cluster", [1, 2, 4])
+@pytest.mark.parametrize("weighted", [False, True], ids=["plain", "weighted"])
+def test_dispersion_by_product_of_eviction(orc, keys, cluster, weighted, monkeypatch):
+    """sigma from the eviction's own score pass: the pre-eviction rows of
+    every unit that evicted, untouched elsewhere; the eviction itself is
+    unchanged by asking for it."""
+    monkeypatch.setenv("VD_CLUSTER_SIZE", str(cluster))
+    d, N, B = 128, 300, 64
+    lens = [N + B, N + 5, 100]
+    cache = filled(3, 2, 2, N + B, d, lens, seed=61 + cluster, gen="student_t")
+    ref = vd.Cache(cache.k.clone(), cache.v.clone(), cache.len.clone())
+    pre = bits(units_view(cache.k if keys else cache.v))
+    attn = None
+    if weighted:
+        g = torch.Generator(device="cuda").manual_seed(9)
+        attn = torch.rand(cache.unit_shape() + (N + B,), generator=g, device="cuda") * 0.9
+    out = torch.full(cache.unit_shape(), -1.0, device="cuda")
+    ka = torch.empty(cache.unit_shape() + (N,), dtype=torch.int32, device="cuda")
+    kb = torch.empty_like(ka)
+    vd.vd_evict_block_ex(cache, N, score_keys=keys, attn=attn, kept_idx_out=ka,
+                         dispersion_out=out)
+    vd.vd_evict_block_ex(ref, N, score_keys=keys, attn=attn, kept_idx_out=kb)
+    assert vd.vd_get_device_status() == 0
+    assert torch.equal(ka, kb)
+    assert torch.equal(cache.k, ref.k) and torch.equal(cache.v, ref.v)
+    got = out.view(-1).cpu().numpy()
+    for u in range(cache.units):
+        n = lens[u // 4]
+        if n <= N:
+            assert got[u] == -1.0
+            continue
+        want = orc.dispersion(pre[u, :n])
+        assert abs(got[u] - want) <= 1e-5 * want + 1e-6, (u, got[u], want)
+
+
+@pytest.mark.parametrize("cluster", [1, 4])
+def test_dispersion_by_product_running_mean(orc, cluster, monkeypatch):
+    """With the running-sum mean (S / n) the by-product is the same sigma."""
+    monkeypatch.setenv("VD_CLUSTER_SIZE", str(cluster))
+    d, N, B = 256, 400, 48
+    cache = filled(2, 1, 2, N + B, d, [N, N], seed=71 + cluster)
+    rs = torch.empty(cache.unit_shape() + (d,), dtype=torch.float64, device="cuda")
+    vd.vd_running_sum_init(cache, rs)
+    cache.len.fill_(N + B)                  # the next B rows were already written
+    pre = bits(units_view(cache.v))
+    out = torch.full(cache.unit_shape(), -1.0, device="cuda")
+    vd.vd_evict_block_ex(cache, N, None, B, vd.VD_SCORE_L2, vd.VD_MU_RUNNING, rs,
+                         dispersion_out=out)
+    assert vd.vd_get_device_status() == 0
+    got = out.view(-1).cpu().numpy()
+    for u in range(cache.units):
+        want = orc.dispersion(pre[u, :N + B])
+        assert abs(got[u] - want) <= 1e-5 * want + 1e-6, (u, got[u], want)
+
+
 def test_option_errors():
     cache = filled(1, 1, 1, 64, 64, [64], seed=1)
     rs = torch.zeros(1, 1, 1, 64, dtype=torch.float64, device="cuda")
@@ -154,6 +210,10 @@ def test_option_errors():
         vd.vd_score_ex(cache, vd.VD_SCORE_DIR, False, None,
                        torch.zeros(1, 1, 1, device="cuda"))
     assert e.value.code == 1                  # sigma is defined on L2 distances
+    with pytest.raises(vd.VdError) as e:
+        vd.vd_evict_block_ex(cache, 32, variant=vd.VD_SCORE_NORM,
+                             dispersion_out=torch.zeros(1, 1, 1, device="cuda"))
+    assert e.value.code == 1
     attn = torch.full((1, 1, 1, 64), 0.5, device="cuda")
     attn[..., 3] = 1.0                        # a weight of 1: infinite factor
     vd.vd_evict_block_ex(cache, 32, attn=attn)
