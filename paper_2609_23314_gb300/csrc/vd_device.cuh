@@ -40,6 +40,42 @@ __device__ __forceinline__ void unpack8(const uint4& q, float (&x)[8]) {
   x[7] = __uint_as_float(q.w & 0xffff0000u);
 }
 
+// ---------------------------------------------------------------------------
+// Packed fp32 pairs: the sm_100-family f32x2 add/fma instructions do two
+// fp32 operations (each rounded as the scalar one) per issue slot.  A pair
+// is a 64-bit register: low half = first element, high half = second.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ unsigned long long f2_pack(float lo, float hi) {
+  unsigned long long r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
+  return r;
+}
+
+__device__ __forceinline__ float f2_hsum(unsigned long long v) {
+  float lo, hi;
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
+  return lo + hi;
+}
+
+__device__ __forceinline__ unsigned long long f2_sub(unsigned long long a, unsigned long long b) {
+  unsigned long long r;
+  asm("sub.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
+  return r;
+}
+
+__device__ __forceinline__ unsigned long long f2_fma(unsigned long long a, unsigned long long b,
+                                                     unsigned long long c) {
+  unsigned long long r;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(r) : "l"(a), "l"(b), "l"(c));
+  return r;
+}
+
+// Two bf16 values (one 32-bit word, first element in the low half) widened
+// to a packed fp32 pair.
+__device__ __forceinline__ unsigned long long bf16x2_to_f2(uint32_t w) {
+  return f2_pack(__uint_as_float(w << 16), __uint_as_float(w & 0xffff0000u));
+}
+
 __device__ __forceinline__ uint4 ld_cg16(const void* p) {
   uint4 r;
   asm volatile("ld.global.cg.v4.u32 {%0,%1,%2,%3}, [%4];"

@@ -50,13 +50,22 @@
 
 namespace vd {
 
-// cp.async ring: kRingStages stages of kRingItems 16-byte copies per thread
-// (overridable at build time for tuning sweeps).
+// cp.async rings: STAGES stages of ITEMS 16-byte copies per thread.  The
+// block kernels (which also hold keys and slot lists in shared memory) and
+// the decode / score-only kernels (which hold neither, so they can afford a
+// deeper ring) have their own shapes; overridable at build time for tuning
+// sweeps.
 #ifndef VD_RING_STAGES
 #define VD_RING_STAGES 4
 #endif
 #ifndef VD_RING_ITEMS
 #define VD_RING_ITEMS 2
+#endif
+#ifndef VD_DECODE_RING_STAGES
+#define VD_DECODE_RING_STAGES VD_RING_STAGES
+#endif
+#ifndef VD_DECODE_RING_ITEMS
+#define VD_DECODE_RING_ITEMS VD_RING_ITEMS
 #endif
 // Resident CTAs per SM the block and decode kernels are compiled for (caps
 // registers per thread at 65536 / (256 * n)).
@@ -66,9 +75,20 @@ namespace vd {
 #ifndef VD_DECODE_MIN_CTAS
 #define VD_DECODE_MIN_CTAS 4
 #endif
-constexpr int kRingStages = VD_RING_STAGES;
-constexpr int kRingItems = VD_RING_ITEMS;
-constexpr int kRingBytes = kRingStages * kRingItems * kThreads * 16;
+template <int STAGES, int ITEMS>
+struct RingShape {
+  static constexpr int kStages = STAGES;
+  static constexpr int kItems = ITEMS;
+  static constexpr int kBytes = STAGES * ITEMS * kThreads * 16;
+};
+using BlockRing = RingShape<VD_RING_STAGES, VD_RING_ITEMS>;
+using DecodeRing = RingShape<VD_DECODE_RING_STAGES, VD_DECODE_RING_ITEMS>;
+
+// Ring bytes of a launch: block eviction (with the select) or decode /
+// score-only.
+__host__ __device__ constexpr int ring_bytes(bool with_select) {
+  return with_select ? BlockRing::kBytes : DecodeRing::kBytes;
+}
 
 struct EvictArgs {
   uint16_t* k;            // bf16 [U][capacity][d]
@@ -135,7 +155,7 @@ struct SmemLayout {
 __host__ __device__ inline SmemLayout smem_layout(int capacity, int cluster, bool with_select) {
   SmemLayout l;
   l.ring = (sizeof(Smem) + 127) & ~(size_t)127;
-  l.keys = l.ring + kRingBytes;
+  l.keys = l.ring + (size_t)ring_bytes(with_select);
   const size_t rows = with_select ? (size_t)((capacity + cluster - 1) / cluster) : 0;
   l.perm = l.keys + align16(rows * 4);
   l.total = l.perm + (with_select ? align16((size_t)capacity * 2) : 0);
@@ -149,7 +169,7 @@ __host__ __device__ inline SmemLayout smem_layout(int capacity, int cluster, boo
 // same number of steps, so consume() may use warp shuffles; it receives every
 // item slot with `in` = item < count and the chunk (zeros for idle lanes).
 // A thread only reuses a ring slot after its own consume() used the data.
-template <class RowOf, class Consume>
+template <class Ring, class RowOf, class Consume>
 __device__ __forceinline__ void stream_rows(const uint16_t* __restrict__ base, int d, int chunk0,
                                             int nchunks, int P, int count, RowOf row_of,
                                             Consume consume, uint32_t ring) {
@@ -157,6 +177,7 @@ __device__ __forceinline__ void stream_rows(const uint16_t* __restrict__ base, i
   const int ci = lane & (P - 1);
   const bool active = ci < nchunks;
   const int ng = kThreads / P, g = tid / P;
+  constexpr int kRingStages = Ring::kStages, kRingItems = Ring::kItems;
   const int per_stage = ng * kRingItems;
   const int nst = count > 0 ? (count + per_stage - 1) / per_stage : 0;
   const uint32_t my = ring + (uint32_t)tid * 16u;
@@ -191,6 +212,106 @@ __device__ __forceinline__ void stream_rows(const uint16_t* __restrict__ base, i
   cp_async_wait<0>();
 }
 
+// Squared norm of one 16-byte chunk (8 bf16 values) of a row: of v - mean
+// for VAR 0 (m2: the chunk's mean as packed pairs), of v itself for VAR 2.
+template <int VAR>
+__device__ __forceinline__ float chunk_sq(const uint4& q, const unsigned long long (&m2)[4]) {
+  const uint32_t w[4] = {q.x, q.y, q.z, q.w};
+  unsigned long long acc = 0ull;
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    const unsigned long long x = bf16x2_to_f2(w[k]);
+    if (VAR == 0) {
+      const unsigned long long dv = f2_sub(x, m2[k]);
+      acc = f2_fma(dv, dv, acc);
+    } else {
+      acc = f2_fma(x, x, acc);
+    }
+  }
+  return f2_hsum(acc);
+}
+
+// Score pass over R contiguous rows (row stride d = 8 * LPR elements, LPR in
+// {8, 16, 32} lanes per row) for the L2 (VAR 0) and Norm (VAR 2) rules.
+// Rows stream through the thread-private cp.async ring; each lane keeps its
+// chunk's partial sums for a batch of kBatch rows and the LPR lanes of a row
+// group reduce the batch with a transposed butterfly (kBatch - 1 exchanges
+// for kBatch rows, then log2(LPR / kBatch) plain steps), after which lane
+// ci holds row ci / (LPR / kBatch) of the batch: the lanes with
+// ci % (LPR / kBatch) == 0 call finish(j, s) for the batch's valid rows (j is
+// the row's index in [0, R)).  Same arithmetic per element as the general
+// path; only the order of the fp32 additions differs.
+template <int VAR, int LPR, class Ring, class Finish>
+__device__ __forceinline__ void score_rows_fast(const uint16_t* __restrict__ rows, int R,
+                                                const float* mu, Finish finish, uint32_t ring) {
+  constexpr int kStages = Ring::kStages, kItems = Ring::kItems;
+  constexpr int kBatch = 8;
+  static_assert(kBatch % kItems == 0 && LPR >= kBatch, "batch shape");
+  constexpr int kStagesPerBatch = kBatch / kItems;
+  constexpr int kGroups = kThreads / LPR;
+  constexpr int kD = LPR * 8;
+  constexpr int kSpread = LPR / kBatch;  // lanes per row after the transposed steps
+  const int tid = threadIdx.x, lane = tid & 31, ci = lane & (LPR - 1), g = tid / LPR;
+  unsigned long long m2[4];
+#pragma unroll
+  for (int k = 0; k < 4; ++k)
+    m2[k] = VAR == 0 ? f2_pack(mu[ci * 8 + 2 * k], mu[ci * 8 + 2 * k + 1]) : 0ull;
+  const int per_stage = kGroups * kItems;
+  const int nst = (R + per_stage - 1) / per_stage;
+  const uint32_t my = ring + (uint32_t)tid * 16u;
+  const uint16_t* p0 = rows + (size_t)g * kD + ci * 8;
+  auto slot = [&](int s, int u) {
+    return my + (uint32_t)((s * kItems + u) * kThreads * 16);
+  };
+  auto issue = [&](int st) {
+    if (st < nst) {
+#pragma unroll
+      for (int u = 0; u < kItems; ++u) {
+        const int k = st * kItems + u;  // this group's k-th row: g + k * kGroups
+        if (g + k * kGroups < R) cp_async16(slot(st % kStages, u), p0 + (size_t)k * kGroups * kD);
+      }
+    }
+    cp_async_commit();
+  };
+  for (int st = 0; st < kStages; ++st) issue(st);
+  const int nbatch = (nst + kStagesPerBatch - 1) / kStagesPerBatch;
+  for (int b = 0; b < nbatch; ++b) {
+    float part[kBatch];
+#pragma unroll
+    for (int sb = 0; sb < kStagesPerBatch; ++sb) {
+      const int st = b * kStagesPerBatch + sb;
+      cp_async_wait<kStages - 1>();
+#pragma unroll
+      for (int u = 0; u < kItems; ++u) {
+        const int k = st * kItems + u;
+        uint4 q = make_uint4(0u, 0u, 0u, 0u);
+        if (g + k * kGroups < R) q = ld_shared16(slot(st % kStages, u));
+        part[sb * kItems + u] = chunk_sq<VAR>(q, m2);
+      }
+      issue(st + kStages);
+    }
+    // transposed steps over lane offsets LPR/2, LPR/4, LPR/8
+#pragma unroll
+    for (int j = 0; j < 3; ++j) {
+      const int h = kBatch >> (j + 1), off = LPR >> (j + 1);
+      const bool upper = (ci & off) != 0;
+#pragma unroll
+      for (int k = 0; k < h; ++k) {
+        const float send = upper ? part[k] : part[k + h];
+        const float keep = upper ? part[k + h] : part[k];
+        part[k] = keep + __shfl_xor_sync(kFull, send, off);
+      }
+    }
+#pragma unroll
+    for (int off = kSpread / 2; off >= 1; off >>= 1) part[0] += __shfl_xor_sync(kFull, part[0], off);
+    if (ci % kSpread == 0) {
+      const int j = g + (b * kBatch + ci / kSpread) * kGroups;
+      if (j < R) finish(j, sqrtf(part[0]));
+    }
+  }
+  cp_async_wait<0>();
+}
+
 // Merges every thread's double-float column partials (8 columns from column
 // `col`, lanes grouped P per row) into acc_hi/acc_lo (zeroed by the caller),
 // across the warp with TwoSum shuffles and across warps in a fixed order.
@@ -219,7 +340,7 @@ __device__ __forceinline__ void merge_columns(float (&hi)[8], float (&lo)[8], in
 
 // acc (zeroed here) <- sum over items [0, count) of sign(item) * V[row(item)],
 // restricted to 16-byte column chunks [chunk0, chunk0 + nchunks).
-template <class RowOf, class SignOf>
+template <class Ring, class RowOf, class SignOf>
 __device__ __forceinline__ void sum_rows(const uint16_t* vbase, int d, int chunk0, int nchunks,
                                          int P, int count, RowOf row_of, SignOf sign_of, Smem& S,
                                          uint32_t ring) {
@@ -231,7 +352,7 @@ __device__ __forceinline__ void sum_rows(const uint16_t* vbase, int d, int chunk
   float hi[8], lo[8];
 #pragma unroll
   for (int k = 0; k < 8; ++k) hi[k] = lo[k] = 0.f;
-  stream_rows(vbase, d, chunk0, nchunks, P, count, row_of,
+  stream_rows<Ring>(vbase, d, chunk0, nchunks, P, count, row_of,
               [&](int item, bool in, const uint4& q) {
                 if (in && active) {
                   float x[8];
@@ -461,6 +582,7 @@ __device__ __forceinline__ void cluster_build_perm(const uint32_t* keys, int r0,
 // source row perm[r] (or r + 1 when perm is null: the decode shift).  A
 // source at or above n (impossible for a consistent slot list) is not read
 // and is recorded as kStInternal (its row then holds unspecified bytes).
+template <class Ring>
 __device__ __forceinline__ void compact_slice(uint16_t* kb, uint16_t* vb, int d, int chunk0,
                                               int cps, int r_begin, int r_end, int n,
                                               const uint16_t* perm, unsigned* status,
@@ -472,6 +594,7 @@ __device__ __forceinline__ void compact_slice(uint16_t* kb, uint16_t* vb, int d,
   const int my_ch = chunk0 + tid % cps;
   const int my_off = tid / cps;
   uint16_t* col = my_ch < d8 ? kb + my_ch * 8 : vb + (my_ch - d8) * 8;
+  constexpr int kRingStages = Ring::kStages, kRingItems = Ring::kItems;
   const int tile = rs * kRingItems;
   const int ntiles = r_end > r_begin ? (r_end - r_begin + tile - 1) / tile : 0;
   const uint32_t my = ring + (uint32_t)tid * 16u;
@@ -553,6 +676,8 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
     evict_kernel(const EvictArgs a) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   Smem& S = *reinterpret_cast<Smem*>(smem_raw);
+  using Ring = RingShape<DECODE ? DecodeRing::kStages : BlockRing::kStages,
+                         DECODE ? DecodeRing::kItems : BlockRing::kItems>;
   const int C = a.cluster;
   const bool with_select = !DECODE && !a.score_only;
   const SmemLayout L = smem_layout(a.capacity, C, with_select);
@@ -612,7 +737,7 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
         a.kept_out[(size_t)u * a.N + i] = i < n ? i : -1;
     if (DECODE && a.evicted_out && rank == 0 && tid == 0) a.evicted_out[u] = -1;
     if (a.mu_running && a.B > 0 && vchunks > 0) {
-      sum_rows(vb, d, vchunk0, vchunks, vp, a.B, [&](int i) { return first_new + i; },
+      sum_rows<Ring>(vb, d, vchunk0, vchunks, vp, a.B, [&](int i) { return first_new + i; },
                [](int) { return 1.f; }, S, ring);
       if (tid < vchunks * 8) {
         const int c = vchunk0 * 8 + tid;
@@ -638,7 +763,7 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
       p0 = r0;
       p1 = r1;
     }
-    sum_rows(sb, d, 0, d8, lpr, max(0, p1 - p0), [&](int i) { return p0 + i; },
+    sum_rows<Ring>(sb, d, 0, d8, lpr, max(0, p1 - p0), [&](int i) { return p0 + i; },
              [](int) { return 1.f; }, S, ring);
     if (C > 1) cluster_sync(); else __syncthreads();
     if (tid < d) {
@@ -693,7 +818,47 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
     unsigned best_key = 0xffffffffu;   // hole-fill: key of this thread's minimum
     int best_slot = -1;
     float* sc_out = a.scores_out ? a.scores_out + (size_t)u * a.capacity : nullptr;
-    stream_rows(
+    // everything a row's score feeds: the output, sigma, its key
+    auto finish_row = [&](int item, float s) {
+      const int r = r0 + item;
+      if (sc_out && !weighted) sc_out[r] = s;
+      if (VAR == 0 && disp) {  // sum s and s^2 (the square split exactly by an FMA)
+        ff_accumulate(ds_hi, ds_lo, s);
+        const float q2 = s * s;
+        ff_accumulate(dq_hi, dq_lo, q2);
+        dq_lo += fmaf(s, s, -q2);
+      }
+      if (!a.score_only) {
+        bool bad;
+        const uint32_t key = score_key(s, bad);
+        if (bad) record_status(a.status, kStNonfinite);
+        if (DECODE) {
+          // lowest score first; among equal scores the latest token
+          // (highest slot, or highest position in the hole-fill layout,
+          // whose positions are read only to settle an exact tie)
+          if constexpr (!HF) {
+            const unsigned long long pk = ((unsigned long long)key << 32) |
+                                          (unsigned long long)(0xffffffffu - (unsigned)r);
+            best = pk < best ? pk : best;
+          } else if (key < best_key || (key == best_key && pos_of(r) > pos_of(best_slot))) {
+            best_key = key;
+            best_slot = r;
+          }
+        } else {
+          keys[item] = key;
+        }
+      }
+    };
+    const uint16_t* rows = sb + (size_t)r0 * d;
+    bool fast = false;
+    if constexpr (VAR != 1) {  // head dims 64, 128, 256: one 16-byte chunk per lane
+      fast = true;
+      if (d == 128) score_rows_fast<VAR, 16, Ring>(rows, r1 - r0, S.mu, finish_row, ring);
+      else if (d == 256) score_rows_fast<VAR, 32, Ring>(rows, r1 - r0, S.mu, finish_row, ring);
+      else if (d == 64) score_rows_fast<VAR, 8, Ring>(rows, r1 - r0, S.mu, finish_row, ring);
+      else fast = false;
+    }
+    if (!fast) stream_rows<Ring>(
         sb, d, 0, d8, lpr, r1 - r0, [&](int i) { return r0 + i; },
         [&](int item, bool in, const uint4& q) {
           float x[8];
@@ -729,37 +894,7 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
             for (int off = 1; off < lpr; off <<= 1) acc += __shfl_xor_sync(kFull, acc, off);
             s = (nv > 0.f && !mu_zero) ? 0.5f * acc : 1.f;
           }
-          if (in && ci == 0) {
-            const int r = r0 + item;
-            if (sc_out && !weighted) sc_out[r] = s;
-            if (VAR == 0 && disp) {  // sum s and s^2 (the square split exactly by an FMA)
-              ff_accumulate(ds_hi, ds_lo, s);
-              const float q2 = s * s;
-              ff_accumulate(dq_hi, dq_lo, q2);
-              dq_lo += fmaf(s, s, -q2);
-            }
-            if (!a.score_only) {
-              bool bad;
-              const uint32_t key = score_key(s, bad);
-              if (bad) record_status(a.status, kStNonfinite);
-              if (DECODE) {
-                // lowest score first; among equal scores the latest token
-                // (highest slot, or highest position in the hole-fill layout,
-                // whose positions are read only to settle an exact tie)
-                if constexpr (!HF) {
-                  const unsigned long long pk = ((unsigned long long)key << 32) |
-                                                (unsigned long long)(0xffffffffu - (unsigned)r);
-                  best = pk < best ? pk : best;
-                } else if (key < best_key ||
-                           (key == best_key && pos_of(r) > pos_of(best_slot))) {
-                  best_key = key;
-                  best_slot = r;
-                }
-              } else {
-                keys[item] = key;
-              }
-            }
-          }
+          if (in && ci == 0) finish_row(item, s);
         },
         ring);
     // sigma is defined on the L2 distance (VAR 0), whose scores never read
@@ -893,7 +1028,7 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
   // the evicted rows are read again.
   if (a.mu_running && vchunks > 0) {
     const int B = VAR != 2 ? 0 : a.B;
-    sum_rows(vb, d, vchunk0, vchunks, vp, B + (n - Nb),
+    sum_rows<Ring>(vb, d, vchunk0, vchunks, vp, B + (n - Nb),
              [&](int i) {
                const int r =
                    i < B ? first_new + i : (DECODE ? e_first : (int)perm[Nb + (i - B)]);
@@ -912,7 +1047,7 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
 
   // ---- 6. in-place compaction of this CTA's column slice ---------------
   if constexpr (!HF) {
-    compact_slice(kb, vb, d, chunk0, cps, e_first, Nb, n, DECODE ? nullptr : perm, a.status,
+    compact_slice<Ring>(kb, vb, d, chunk0, cps, e_first, Nb, n, DECODE ? nullptr : perm, a.status,
                   ring);
   } else {
     // hole-fill: the kept rows at or above N move into the evicted slots
