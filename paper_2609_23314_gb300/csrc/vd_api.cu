@@ -215,17 +215,21 @@ bool cluster_allowed(int c, int d) {
   return c == 1 || (total_chunks % c == 0 && total_chunks / c >= 4);
 }
 
-// CTAs per unit: the smallest C in {1, 2, 4, 8, 16} that keeps row segments
-// of at least 64 bytes of [K | V] and whose CTAs either form one nearly full
-// wave (>= 85% of the resident slots at that C's shared-memory size) or at
-// least two waves, so that no short tail wave runs alone; with none such,
-// the largest allowed C.  (Measured on GB300: a 1.1-wave launch loses ~15%,
-// while larger clusters than needed pay for extra synchronisation and
-// narrower row segments.)  want (VD_CLUSTER_SIZE: 1, 2, 4, 8 or 16)
-// overrides the choice, for tuning.
+// CTAs per unit: C in {1, 2, 4, 8, 16}, keeping row segments of at least 64
+// bytes of [K | V].  Waves = CTAs / resident slots at that C's shared-memory
+// size.  Decode and score-only launches: the smallest C whose CTAs form one
+// nearly full wave (0.85-1) or at least two waves, so that no short tail
+// wave runs alone.  Ordered block eviction (moves most of the cache): the
+// smallest C with 0.85-1 waves or at least four, else the decode rule.
+// Hole-fill block eviction (moves few rows, so the select's cluster
+// synchronisation dominates and grows with C): the smallest C with at least
+// 0.85 of a wave.  With none such, the largest allowed C.  (Measured on
+// GB300: prefill_wide ordered C=8 (4.4 waves) 0.574 ms vs C=4 (2.2) 0.586;
+// hole-fill C=2 (1.1 waves) 0.205 vs C=4 0.216; decode C=1.)  want
+// (VD_CLUSTER_SIZE: 1, 2, 4, 8 or 16) overrides the choice, for tuning.
 int choose_cluster(const void* kern, long long units, int d, int capacity, bool with_select,
-                   int want, const DeviceState& st, size_t* smem_out) {
-  int chosen = 0, largest = 1;
+                   bool holefill, int want, const DeviceState& st, size_t* smem_out) {
+  int chosen = 0, fallback = 0, largest = 1;
   for (int c = 1; c <= 16; c *= 2) {
     if (want >= 1 && c != want) continue;
     if (want < 1 && !cluster_allowed(c, d)) continue;
@@ -240,19 +244,30 @@ int choose_cluster(const void* kern, long long units, int d, int capacity, bool 
     if (occ < 1 || !cluster_fits(kern, units, c, smem)) continue;
     largest = c;
     const double waves = (double)(units * c) / ((double)st.sms * occ);
-    if (want >= 1 || (waves >= 0.85 && waves <= 1.0) || waves >= 2.0) {
+    const bool full_wave = waves >= 0.85 && waves <= 1.0;
+    bool ok;
+    if (want >= 1)
+      ok = true;
+    else if (with_select && holefill)
+      ok = waves >= 0.85;
+    else if (with_select)
+      ok = full_wave || waves >= 4.0;
+    else
+      ok = full_wave || waves >= 2.0;
+    if (ok) {
       chosen = c;
       break;
     }
+    if (fallback == 0 && (full_wave || waves >= 2.0)) fallback = c;
   }
-  if (chosen == 0) chosen = largest;
+  if (chosen == 0) chosen = fallback ? fallback : largest;
   *smem_out = vd::smem_layout(capacity, chosen, with_select).total;
   return chosen;
 }
 
 // choose_cluster, remembered per launch shape.
 int cached_cluster(const void* kern, long long units, int d, int capacity, bool with_select,
-                   DeviceState& st, size_t* smem_out) {
+                   bool holefill, DeviceState& st, size_t* smem_out) {
   const char* env = std::getenv("VD_CLUSTER_SIZE");
   const int want = env ? std::atoi(env) : 0;
   const int ws = with_select ? 1 : 0;
@@ -267,7 +282,8 @@ int cached_cluster(const void* kern, long long units, int d, int capacity, bool 
       }
     }
   }
-  const int c = choose_cluster(kern, units, d, capacity, with_select, want, st, smem_out);
+  const int c = choose_cluster(kern, units, d, capacity, with_select, holefill, want, st,
+                               smem_out);
   std::lock_guard<std::mutex> lk(g_mu);
   st.choice[st.next_choice] = ClusterChoice{kern, units, d, capacity, ws, want, c, *smem_out};
   st.next_choice = (st.next_choice + 1) % kChoiceSlots;
@@ -355,7 +371,7 @@ vd_status run(const vd_cache* c, int32_t N, const int32_t* N_dev, int32_t B, vd_
   a.weights = weights;
   a.disp_out = disp_out;
   size_t smem = 0;
-  a.cluster = cached_cluster(kern, units, c->head_dim, c->capacity, !small, *st, &smem);
+  a.cluster = cached_cluster(kern, units, c->head_dim, c->capacity, !small, holefill, *st, &smem);
   if (smem > (size_t)st->smem_optin) return VD_ERR_UNSUPPORTED;
 
   r = launch(kern, units, a.cluster, smem, a, s);
