@@ -213,6 +213,43 @@ def test_decode_steps_running_sum(orc, var):
 
 
 # ---------------------------------------------------------------------------
+# block then decode events at head dims with the batched score pass (64, 256)
+# and without it (96), ragged batch tails, both mean modes
+# ---------------------------------------------------------------------------
+@pytest.mark.parametrize("var", VARS, ids=VAR_IDS)
+@pytest.mark.parametrize("d", [64, 96, 256])
+@pytest.mark.parametrize("mu", [vd.VD_MU_RECOMPUTE, vd.VD_MU_RUNNING], ids=["recompute", "running"])
+def test_block_then_decode_head_dims(orc, var, d, mu):
+    N, B = 150, 37                      # B and the lengths are not multiples of a batch
+    lens = [N + B, N + 1, N + 20]
+    cache = filled_cache(3, 2, 2, N + B, d, lens, seed=d + 7 * mu, gen="student_t")
+    rs = None
+    if mu == vd.VD_MU_RUNNING:
+        rs = torch.zeros(cache.unit_shape() + (d,), dtype=torch.float64, device="cuda")
+        cache.len.copy_(torch.tensor([x - B for x in lens], dtype=torch.int32))
+        vd.vd_running_sum_init(cache, rs)
+        cache.len.copy_(torch.tensor(lens, dtype=torch.int32))
+    for c in (None, 2):
+        if c is not None and 2 * (d // 8) % c:
+            continue
+        work = vd.Cache(cache.k.clone(), cache.v.clone(), cache.len.clone())
+        wrs = rs.clone() if rs is not None else None
+        with cluster_size(c):
+            evict_and_check(orc, work, N, B, var, mu, wrs)
+            # one decode step on the compacted cache
+            st = wl.TokenStream("student_t", work.units, d, device="cuda", seed=d + 1)
+            k, v = st.next(1)
+            us = work.unit_shape()
+            vd.vd_append(work, k.view(us + (1, d)).contiguous(), v.view(us + (1, d)).contiguous(), 1)
+            evict_and_check(orc, work, N, 1, var, mu, wrs, decode=True)
+        if wrs is not None:
+            ref = torch.zeros_like(wrs)
+            vd.vd_running_sum_init(work, ref)
+            scale = units_view(work.v).float().abs().sum(dim=1).max().item()
+            assert torch.max(torch.abs(ref - wrs)).item() <= 1e-12 * scale
+
+
+# ---------------------------------------------------------------------------
 # ties, duplicates, degenerate caches, N extremes, poisoned tails
 # ---------------------------------------------------------------------------
 @pytest.mark.parametrize("var", VARS, ids=VAR_IDS)
