@@ -305,20 +305,15 @@ class Prefill:
             ev[1].record()
 
     def moved_rows(self, kept_list):
-        """Rows moved per launch, all units: ordered layout, N - first evicted
-        slot per unit; hole-fill layout, the refilled slots (kept[r] != r)."""
+        """Rows moved per launch, all units: the slots r < N that received
+        another row (kept[r] not r, and not -1).  Ordered layout: N - the first
+        evicted slot of every unit that evicted; hole-fill: the refilled slots."""
         t = self.torch
         total = 0
         ar = t.arange(self.N, device=self.device, dtype=t.int32)
         for kp in kept_list:
             kk = kp.view(self.U, self.N)
-            same = (kk == ar)
-            if self.holefill:
-                total += int((~same).sum().item())
-                continue
-            first = t.where(same.all(dim=1), t.full((self.U,), self.N, device=self.device),
-                            (~same).int().argmax(dim=1))
-            total += int((self.N - first).sum().item())
+            total += int(((kk != ar) & (kk >= 0)).sum().item())
         return total / max(1, len(kept_list))
 
     def bytes_per_launch(self, moved_rows_total):
@@ -457,10 +452,11 @@ class Decode:
         below N."""
         total = 0
         for e in evicted_list:
+            e = e.long()
             if self.holefill:
-                total += int((e < self.N).sum().item())
-            else:
-                total += int((self.N - e.long()).sum().item())
+                total += int(((e >= 0) & (e < self.N)).sum().item())
+            else:  # slots e .. N-1 shift down by one; -1: nothing evicted
+                total += int(self.torch.where(e >= 0, self.N - e, 0).sum().item())
         return total / max(1, len(evicted_list))
 
     def bytes_per_launch(self, moved_rows_total):

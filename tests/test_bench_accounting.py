@@ -1,0 +1,109 @@
+"""The benchmark's host-side accounting (moved rows, algorithmic bytes, the
+ncu traffic lookup) and its CPU reference arm; CPU only."""
+from __future__ import annotations
+
+import contextlib
+import io
+import json
+import os
+import sys
+
+import numpy as np
+import pytest
+import torch
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+sys.path.insert(0, ROOT)
+import bench  # noqa: E402
+
+
+def ordered_kept(n, N, evicted):
+    """Slots kept by an ordered eviction, -1 padded to N."""
+    kept = [r for r in range(n) if r not in evicted][:N]
+    return kept + [-1] * (N - len(kept))
+
+
+def holefill_kept(n, N, evicted):
+    """Slot map of the hole-fill layout: kept rows at or above N fill the
+    evicted slots below N in ascending order; other slots keep their row."""
+    if n <= N:
+        return list(range(n)) + [-1] * (N - n)
+    movers = [r for r in range(N, n) if r not in evicted]
+    holes = [r for r in range(N) if r in evicted]
+    assert len(movers) == len(holes)
+    out = list(range(N))
+    for h, m in zip(holes, movers):
+        out[h] = m
+    return out
+
+
+def fake(cls, U, N, B, d, holefill, mu=1, attn=False):
+    w = object.__new__(cls)
+    w.torch, w.device, w.U, w.N, w.B, w.d = torch, torch.device("cpu"), U, N, B, d
+    w.holefill, w.mu, w.attn = holefill, mu, (object() if attn else None)
+    return w
+
+
+@pytest.mark.parametrize("holefill", [False, True], ids=["ordered", "holefill"])
+def test_prefill_moved_rows(holefill):
+    rng = np.random.default_rng(3)
+    U, N, B = 6, 40, 9
+    w = fake(bench.Prefill, U, N, B, 8, holefill)
+    kept_list, want = [], 0
+    for _ in range(3):
+        rows = []
+        for u in range(U):
+            n = N + B if u != 5 else N - 7           # one unit below budget: nothing moves
+            ev = set(rng.choice(n, size=n - N, replace=False).tolist()) if n > N else set()
+            k = holefill_kept(n, N, ev) if holefill else ordered_kept(n, N, ev)
+            rows.append(k)
+            if n > N:
+                want += len([h for h in ev if h < N]) if holefill else max(0, N - min(ev))
+        kept_list.append(torch.tensor(rows, dtype=torch.int32))
+    assert w.moved_rows(kept_list) == pytest.approx(want / 3)
+
+
+@pytest.mark.parametrize("holefill", [False, True], ids=["ordered", "holefill"])
+def test_decode_moved_rows(holefill):
+    U, N = 5, 30
+    w = fake(bench.Decode, U, N, 1, 8, holefill)
+    e = torch.tensor([0, 7, N, -1, N - 1], dtype=torch.int32)   # N: the new token itself
+    want = (1 + 1 + 0 + 0 + 1) if holefill else (N + (N - 7) + 0 + 0 + 1)
+    assert w.moved_rows([e, e]) == want
+
+
+def test_bytes_per_launch():
+    U, N, B, d = 4, 100, 20, 64
+    w = fake(bench.Prefill, U, N, B, d, False, attn=True)
+    alg, nominal = w.bytes_per_launch(37)
+    v_read = U * (N + B) * d * 2
+    state = U * d * 8 * 2 + U * (N + B) * 4
+    assert alg == v_read + 37 * d * 8 + state
+    assert nominal == v_read + U * N * d * 8 + state
+    wd = fake(bench.Decode, U, N, 1, d, True, mu=0)
+    alg, nominal = wd.bytes_per_launch(3)
+    assert alg == U * (N + 1) * d * 2 + 3 * d * 8 + U * N * 4 + 3 * 4
+    assert nominal == U * (N + 1) * d * 2 + U * d * 8 + U * N * 4 + 3 * 4
+
+
+def test_traffic_is_reported_only_for_the_captured_sources(monkeypatch):
+    with open(os.path.join(ROOT, "profiles", "traffic.json")) as f:
+        t = json.load(f)
+    monkeypatch.setattr(bench, "kernel_source_hash", lambda: t["prefill_wide"]["source_hash"])
+    assert bench.ncu_traffic("prefill_wide") == t["prefill_wide"]["dram_bytes_per_launch"]
+    assert bench.ncu_traffic("no_such_workload") is None
+    monkeypatch.setattr(bench, "kernel_source_hash", lambda: "changed")
+    assert bench.ncu_traffic("prefill_wide") is None
+
+
+def test_reference_arm_runs_on_cpu(monkeypatch):
+    for k in ("WORLD_SIZE", "RANK", "LOCAL_RANK"):
+        monkeypatch.delenv(k, raising=False)
+    out = io.StringIO()
+    with contextlib.redirect_stdout(out):
+        bench.main(["--impl", "reference", "--workload", "tiny_prefill", "--steps", "1",
+                    "--warmup", "3"])
+    line = json.loads(out.getvalue().strip().splitlines()[-1])
+    assert line["impl"] == "reference" and line["value"] > 0 and line["steps"] == 1
+    assert line["cpu_baseline"]["kind"] == "oracle" and line["cpu_baseline"]["cores"] >= 1
+    assert line["e2e"]["h2d_bytes_per_step"] == 0 and line["higher_is_better"] is True
