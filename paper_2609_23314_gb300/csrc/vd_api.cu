@@ -89,7 +89,7 @@ __global__ void __launch_bounds__(kThreads) vd_rsum_init_kernel(const uint16_t* 
     return;
   }
   const uint16_t* vb = v + (size_t)u * cap * d;
-  vd::sum_rows<vd::DecodeRing>(vb, d, 0, d >> 3, lpr, n, [](int i) { return i; },
+  vd::sum_rows<vd::DecodeRing>(0, d >> 3, lpr, n, [&](int i) { return vb + (size_t)i * d; },
                                [](int) { return 1.f; }, S, ring);
   if ((int)threadIdx.x < d)
     rs[(size_t)u * d + threadIdx.x] = (double)S.acc_hi[threadIdx.x] + (double)S.acc_lo[threadIdx.x];

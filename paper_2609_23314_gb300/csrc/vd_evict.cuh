@@ -163,16 +163,15 @@ __host__ __device__ inline SmemLayout smem_layout(int capacity, int cluster, boo
 }
 
 // Streams items [0, count) through a thread-private cp.async ring.  Item i is
-// row row_of(i) of `base` (row stride d elements); in every group of P lanes
-// (P a power of two >= nchunks) lane ci copies 16-byte chunk chunk0 + ci.
+// the row that starts at row_ptr(i); in every group of P lanes (P a power of
+// two >= nchunks) lane ci copies 16-byte chunk chunk0 + ci of it.
 // Thread group g takes items g, g + ng, g + 2 ng, ...  All threads run the
 // same number of steps, so consume() may use warp shuffles; it receives every
 // item slot with `in` = item < count and the chunk (zeros for idle lanes).
 // A thread only reuses a ring slot after its own consume() used the data.
-template <class Ring, class RowOf, class Consume>
-__device__ __forceinline__ void stream_rows(const uint16_t* __restrict__ base, int d, int chunk0,
-                                            int nchunks, int P, int count, RowOf row_of,
-                                            Consume consume, uint32_t ring) {
+template <class Ring, class RowPtr, class Consume>
+__device__ __forceinline__ void stream_rows(int chunk0, int nchunks, int P, int count,
+                                            RowPtr row_ptr, Consume consume, uint32_t ring) {
   const int tid = threadIdx.x, lane = tid & 31;
   const int ci = lane & (P - 1);
   const bool active = ci < nchunks;
@@ -181,7 +180,7 @@ __device__ __forceinline__ void stream_rows(const uint16_t* __restrict__ base, i
   const int per_stage = ng * kRingItems;
   const int nst = count > 0 ? (count + per_stage - 1) / per_stage : 0;
   const uint32_t my = ring + (uint32_t)tid * 16u;
-  const uint16_t* colp = base + (chunk0 + ci) * 8;
+  const int coff = (chunk0 + ci) * 8;
   auto slot = [&](int s, int u) {
     return my + (uint32_t)((s * kRingItems + u) * kThreads * 16);
   };
@@ -190,8 +189,7 @@ __device__ __forceinline__ void stream_rows(const uint16_t* __restrict__ base, i
 #pragma unroll
       for (int u = 0; u < kRingItems; ++u) {
         const int item = g + (st * kRingItems + u) * ng;
-        if (active && item < count)
-          cp_async16(slot(st % kRingStages, u), colp + (size_t)row_of(item) * d);
+        if (active && item < count) cp_async16(slot(st % kRingStages, u), row_ptr(item) + coff);
       }
     }
     cp_async_commit();
@@ -338,12 +336,12 @@ __device__ __forceinline__ void merge_columns(float (&hi)[8], float (&lo)[8], in
   }
 }
 
-// acc (zeroed here) <- sum over items [0, count) of sign(item) * V[row(item)],
-// restricted to 16-byte column chunks [chunk0, chunk0 + nchunks).
-template <class Ring, class RowOf, class SignOf>
-__device__ __forceinline__ void sum_rows(const uint16_t* vbase, int d, int chunk0, int nchunks,
-                                         int P, int count, RowOf row_of, SignOf sign_of, Smem& S,
-                                         uint32_t ring) {
+// acc (zeroed here) <- sum over items [0, count) of sign(item) * (the row at
+// row_ptr(item)), restricted to 16-byte column chunks [chunk0, chunk0 +
+// nchunks).
+template <class Ring, class RowPtr, class SignOf>
+__device__ __forceinline__ void sum_rows(int chunk0, int nchunks, int P, int count,
+                                         RowPtr row_ptr, SignOf sign_of, Smem& S, uint32_t ring) {
   S.acc_hi[threadIdx.x] = 0.f;
   S.acc_lo[threadIdx.x] = 0.f;
   __syncthreads();
@@ -352,7 +350,7 @@ __device__ __forceinline__ void sum_rows(const uint16_t* vbase, int d, int chunk
   float hi[8], lo[8];
 #pragma unroll
   for (int k = 0; k < 8; ++k) hi[k] = lo[k] = 0.f;
-  stream_rows<Ring>(vbase, d, chunk0, nchunks, P, count, row_of,
+  stream_rows<Ring>(chunk0, nchunks, P, count, row_ptr,
               [&](int item, bool in, const uint4& q) {
                 if (in && active) {
                   float x[8];
@@ -696,6 +694,8 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
   uint16_t* kb = a.k + ubase;
   uint16_t* vb = a.v + ubase;
   const uint16_t* sb = a.score_k ? kb : vb;  // rows the mean and the scores come from
+  auto vrow = [&](int r) -> const uint16_t* { return vb + (size_t)r * d; };
+  auto srow = [&](int r) -> const uint16_t* { return sb + (size_t)r * d; };
 
   // ---- validation: uniform across the cluster (per-sequence values only) ---
   if (n < 0 || n > a.capacity || (a.mu_running && !a.score_only && a.B > n)) {
@@ -737,7 +737,7 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
         a.kept_out[(size_t)u * a.N + i] = i < n ? i : -1;
     if (DECODE && a.evicted_out && rank == 0 && tid == 0) a.evicted_out[u] = -1;
     if (a.mu_running && a.B > 0 && vchunks > 0) {
-      sum_rows<Ring>(vb, d, vchunk0, vchunks, vp, a.B, [&](int i) { return first_new + i; },
+      sum_rows<Ring>(vchunk0, vchunks, vp, a.B, [&](int i) { return vrow(first_new + i); },
                [](int) { return 1.f; }, S, ring);
       if (tid < vchunks * 8) {
         const int c = vchunk0 * 8 + tid;
@@ -763,8 +763,8 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
       p0 = r0;
       p1 = r1;
     }
-    sum_rows<Ring>(sb, d, 0, d8, lpr, max(0, p1 - p0), [&](int i) { return p0 + i; },
-             [](int) { return 1.f; }, S, ring);
+    sum_rows<Ring>(0, d8, lpr, max(0, p1 - p0), [&](int i) { return srow(p0 + i); },
+                   [](int) { return 1.f; }, S, ring);
     if (C > 1) cluster_sync(); else __syncthreads();
     if (tid < d) {
       ff t{0.f, 0.f};
@@ -859,7 +859,7 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
       else fast = false;
     }
     if (!fast) stream_rows<Ring>(
-        sb, d, 0, d8, lpr, r1 - r0, [&](int i) { return r0 + i; },
+        0, d8, lpr, r1 - r0, [&](int i) { return srow(r0 + i); },
         [&](int item, bool in, const uint4& q) {
           float x[8];
           unpack8(q, x);
@@ -1028,13 +1028,13 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
   // the evicted rows are read again.
   if (a.mu_running && vchunks > 0) {
     const int B = VAR != 2 ? 0 : a.B;
-    sum_rows<Ring>(vb, d, vchunk0, vchunks, vp, B + (n - Nb),
+    sum_rows<Ring>(vchunk0, vchunks, vp, B + (n - Nb),
              [&](int i) {
                const int r =
                    i < B ? first_new + i : (DECODE ? e_first : (int)perm[Nb + (i - B)]);
-               if ((unsigned)r < (unsigned)n) return r;
+               if ((unsigned)r < (unsigned)n) return vrow(r);
                record_status(a.status, kStInternal);  // self-check: never expected
-               return 0;
+               return vrow(0);
              },
              [&](int i) { return i < B ? 1.f : -1.f; }, S, ring);
     if (tid < vchunks * 8) {
