@@ -124,6 +124,29 @@ vd_status vd_evict_block(const vd_cache* c, int32_t N, const int32_t* N_dev, int
                          vd_variant var, vd_mu_mode mu, double* running_sum,
                          int32_t* kept_idx_out, float* scores_out, vd_stream_t stream);
 
+/* One step of block prompt processing (Sec. 2.2, Eq. block_processing:
+ * C_i = pi_N([C_{i-1} || block_i])) in a single launch: the same result as
+ * vd_append(c, k_new, v_new, B) followed by vd_evict_block(c, N, N_dev, B,
+ * var, mu, running_sum, kept_idx_out, scores_out) -- the same kept slots,
+ * scores, compacted K/V bytes in slots [0, new len), running sum and len --
+ * but the new rows are read straight from the caller's buffers, and only
+ * the ones that survive are written into the cache (appended rows that are
+ * evicted at once are never stored).  Ordered layout, block path.
+ *   k_new, v_new  bf16 device [n_seq][n_layer][n_kv_head][B][head_dim],
+ *                 16-byte aligned, read only; B >= 1.
+ *   len           on entry the rows already cached (the new ones excluded);
+ *                 on exit min(len + B, N_s) -- or len + B where no eviction
+ *                 happens.
+ *   running_sum   (VD_MU_RUNNING) on entry the sum of rows [0, len), on exit
+ *                 the sum of rows [0, new len).
+ * Other arguments as in vd_evict_block.  A sequence with len + B > capacity
+ * is left untouched and records VD_ERR_DEVICE_LEN.  Slots at or above the new
+ * len hold unspecified bytes. */
+vd_status vd_append_evict_block(const vd_cache* c, const void* k_new, const void* v_new,
+                                int32_t B, int32_t N, const int32_t* N_dev, vd_variant var,
+                                vd_mu_mode mu, double* running_sum, int32_t* kept_idx_out,
+                                float* scores_out, vd_stream_t stream);
+
 /* Decode-step eviction (per-token eviction of the abstract and the Sec. 4
  * protocol; Eq. block_processing with B = 1): the caller has appended one
  * token, so len <= N_s + 1.  Units with len = N_s + 1 evict exactly one token

@@ -21,6 +21,7 @@ import threading
 __all__ = [
     "VD_SCORE_L2", "VD_SCORE_DIR", "VD_SCORE_NORM", "VD_MU_RECOMPUTE", "VD_MU_RUNNING",
     "VdError", "Cache", "vd_score", "vd_score_ex", "vd_evict_block", "vd_evict_block_ex",
+    "vd_append_evict_block",
     "vd_evict_decode",
     "vd_evict_block_holefill", "vd_evict_decode_holefill", "vd_append",
     "vd_running_sum_init", "vd_workspace_size", "vd_status_string", "vd_get_device_status",
@@ -67,6 +68,7 @@ def load_library() -> ctypes.CDLL:
             cp = ctypes.POINTER(_VdCache)
             lib.vd_score.argtypes = [cp, S, P, P]
             lib.vd_evict_block.argtypes = [cp, I32, P, I32, S, S, P, P, P, P]
+            lib.vd_append_evict_block.argtypes = [cp, P, P, I32, I32, P, S, S, P, P, P, P]
             lib.vd_evict_decode.argtypes = [cp, I32, P, S, S, P, P, P, P, P]
             lib.vd_evict_block_holefill.argtypes = [cp, I32, P, I32, S, S, P, P, P, P, P, P]
             lib.vd_evict_decode_holefill.argtypes = [cp, I32, P, S, S, P, P, P, P, P, P, P]
@@ -80,6 +82,7 @@ def load_library() -> ctypes.CDLL:
             lib.vd_status_string.restype = ctypes.c_char_p
             lib.vd_get_device_status.argtypes = [P]
             for f in ("vd_score", "vd_score_ex", "vd_evict_block_ex", "vd_evict_block",
+                      "vd_append_evict_block",
                       "vd_evict_decode", "vd_evict_block_holefill",
                       "vd_evict_decode_holefill", "vd_append", "vd_running_sum_init",
                       "vd_get_device_status"):
@@ -186,6 +189,30 @@ def vd_evict_block(cache: Cache, N: int, N_dev=None, B: int = 0, variant: int = 
     _check(load_library().vd_evict_block(cache.ref(), int(N), args[0], int(B), int(variant), int(mu),
                                          args[1], args[2], args[3], _stream(stream)),
            "vd_evict_block")
+
+
+def vd_append_evict_block(cache: Cache, k_new, v_new, B: int, N: int, N_dev=None,
+                          variant: int = VD_SCORE_L2, mu: int = VD_MU_RECOMPUTE,
+                          running_sum=None, kept_idx_out=None, scores_out=None,
+                          stream=None) -> None:
+    """vd_append followed by vd_evict_block in one launch; k_new, v_new: bf16
+    [n_seq, n_layer, n_kv_head, B, head_dim], read straight from the caller's
+    buffers (only surviving rows are written into the cache)."""
+    torch = _torch()
+    us = cache.unit_shape()
+    shape = us + (int(B), cache.head_dim)
+    args = (
+        _ptr(k_new, torch.bfloat16, shape, "k_new", cache.device),
+        _ptr(v_new, torch.bfloat16, shape, "v_new", cache.device),
+        _ptr(N_dev, torch.int32, (cache.n_seq,), "N_dev", cache.device),
+        _ptr(running_sum, torch.float64, us + (cache.head_dim,), "running_sum", cache.device),
+        _ptr(kept_idx_out, torch.int32, us + (int(N),), "kept_idx_out", cache.device),
+        _ptr(scores_out, torch.float32, us + (cache.capacity,), "scores_out", cache.device),
+    )
+    _check(load_library().vd_append_evict_block(cache.ref(), args[0], args[1], int(B), int(N),
+                                                args[2], int(variant), int(mu), args[3],
+                                                args[4], args[5], _stream(stream)),
+           "vd_append_evict_block")
 
 
 def vd_evict_decode(cache: Cache, N: int, N_dev=None, variant: int = VD_SCORE_L2,

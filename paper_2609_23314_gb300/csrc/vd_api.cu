@@ -61,15 +61,21 @@ __global__ void vd_len_add_kernel(int32_t* len, int n_seq, int cap, int B) {
   if (n >= 0 && n <= cap - B) len[s] = n + B;
 }
 
-// Mirrors the eviction kernel's per-sequence decision exactly.
+// Mirrors the eviction kernel's per-sequence decision exactly.  added: the
+// rows a fused append adds to len (0 when they were appended beforehand).
 __global__ void vd_len_clamp_kernel(int32_t* len, const int32_t* N_dev, int N, int n_seq,
-                                    int cap, int B, int running, int decode) {
+                                    int cap, int B, int running, int decode, int added) {
   const int s = blockIdx.x * blockDim.x + threadIdx.x;
   if (s >= n_seq) return;
-  const int n = len[s];
+  const int n0 = len[s];
+  const int n = n0 + added;
   const int Nb = N_dev ? N_dev[s] : N;
-  if (n < 0 || n > cap || (running && B > n)) return;
-  if (Nb < 1 || Nb > N || n <= Nb) return;
+  if (n0 < 0 || n > cap || (running && B > n)) return;
+  if (Nb < 1 || Nb > N) return;
+  if (n <= Nb) {
+    if (added) len[s] = n;
+    return;
+  }
   if (decode && n > Nb + 1) return;
   len[s] = Nb;
 }
@@ -317,7 +323,8 @@ vd_status run(const vd_cache* c, int32_t N, const int32_t* N_dev, int32_t B, vd_
               vd_mu_mode mu, double* running_sum, int32_t* evicted_out, int32_t* kept_idx_out,
               float* scores_out, cudaStream_t s, bool decode, bool score_only,
               int32_t* pos = nullptr, const int32_t* pos_new = nullptr, int score_k = 0,
-              const float* weights = nullptr, float* disp_out = nullptr) {
+              const float* weights = nullptr, float* disp_out = nullptr,
+              const void* k_new = nullptr, const void* v_new = nullptr) {
   vd_status r = validate_cache(c);
   if (r != VD_OK) return r;
   if (var != VD_SCORE_L2 && var != VD_SCORE_DIR && var != VD_SCORE_NORM) return VD_ERR_INVALID_ARG;
@@ -334,6 +341,12 @@ vd_status run(const vd_cache* c, int32_t N, const int32_t* N_dev, int32_t B, vd_
   if (score_k && mu == VD_MU_RUNNING && !score_only) return VD_ERR_UNSUPPORTED;
   const bool holefill = pos != nullptr || pos_new != nullptr;
   if (holefill && (!pos || !pos_new)) return VD_ERR_INVALID_ARG;
+  const bool fused = k_new != nullptr || v_new != nullptr;
+  if (fused) {
+    if (!k_new || !v_new || B < 1 || decode || score_only || holefill) return VD_ERR_INVALID_ARG;
+    if ((reinterpret_cast<uintptr_t>(k_new) | reinterpret_cast<uintptr_t>(v_new)) & 15u)
+      return VD_ERR_ALIGNMENT;
+  }
   DeviceState* st = nullptr;
   r = device_state(&st);
   if (r != VD_OK) return r;
@@ -370,6 +383,8 @@ vd_status run(const vd_cache* c, int32_t N, const int32_t* N_dev, int32_t B, vd_
   a.score_k = score_k ? 1 : 0;
   a.weights = weights;
   a.disp_out = disp_out;
+  a.k_new = static_cast<const uint16_t*>(k_new);
+  a.v_new = static_cast<const uint16_t*>(v_new);
   size_t smem = 0;
   a.cluster = cached_cluster(kern, units, c->head_dim, c->capacity, !small, holefill, *st, &smem);
   if (smem > (size_t)st->smem_optin) return VD_ERR_UNSUPPORTED;
@@ -378,7 +393,8 @@ vd_status run(const vd_cache* c, int32_t N, const int32_t* N_dev, int32_t B, vd_
   if (r != VD_OK || score_only) return r;
   const int threads = 256;
   vd_len_clamp_kernel<<<(c->n_seq + threads - 1) / threads, threads, 0, s>>>(
-      c->len, N_dev, N, c->n_seq, c->capacity, a.B, a.mu_running, decode ? 1 : 0);
+      c->len, N_dev, N, c->n_seq, c->capacity, a.B, a.mu_running, decode ? 1 : 0,
+      fused ? a.B : 0);
   if (cudaGetLastError() != cudaSuccess) return VD_ERR_CUDA;
   return VD_OK;
 }
@@ -393,6 +409,15 @@ extern "C" {
 vd_status vd_score(const vd_cache* c, vd_variant var, float* scores_out, vd_stream_t stream) {
   return run(c, 1, nullptr, 0, var, VD_MU_RECOMPUTE, nullptr, nullptr, nullptr, scores_out,
              reinterpret_cast<cudaStream_t>(stream), false, true);
+}
+
+vd_status vd_append_evict_block(const vd_cache* c, const void* k_new, const void* v_new,
+                                int32_t B, int32_t N, const int32_t* N_dev, vd_variant var,
+                                vd_mu_mode mu, double* running_sum, int32_t* kept_idx_out,
+                                float* scores_out, vd_stream_t stream) {
+  return run(c, N, N_dev, B, var, mu, running_sum, nullptr, kept_idx_out, scores_out,
+             reinterpret_cast<cudaStream_t>(stream), false, false, nullptr, nullptr, 0, nullptr,
+             nullptr, k_new, v_new);
 }
 
 vd_status vd_evict_block(const vd_cache* c, int32_t N, const int32_t* N_dev, int32_t B,

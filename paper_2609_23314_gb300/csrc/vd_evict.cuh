@@ -45,6 +45,7 @@
 
 #include <climits>
 #include <cstdint>
+#include <type_traits>
 
 #include "vd_device.cuh"
 
@@ -115,6 +116,11 @@ struct EvictArgs {
   int32_t score_k;         // 1: mean and scores from K (key-side rules)
   const float* weights;    // nullable [U][capacity]: attention weights a_j (block path)
   float* disp_out;         // nullable [U]: std of the L2 scores of the scored rows
+  // fused append (ordered block path): the B new rows are read from these
+  // staging buffers ([U][B][d] bf16 each) instead of the cache, len does not
+  // count them yet, and only the kept ones are written (nullable: unfused)
+  const uint16_t* k_new;
+  const uint16_t* v_new;
 };
 
 // Fixed part of the dynamic shared memory.  After it (16-byte aligned): the
@@ -584,7 +590,9 @@ template <class Ring>
 __device__ __forceinline__ void compact_slice(uint16_t* kb, uint16_t* vb, int d, int chunk0,
                                               int cps, int r_begin, int r_end, int n,
                                               const uint16_t* perm, unsigned* status,
-                                              uint32_t ring) {
+                                              uint32_t ring, const uint16_t* kn = nullptr,
+                                              const uint16_t* vn = nullptr,
+                                              int first_stage = INT_MAX) {
   const int tid = threadIdx.x;
   const int d8 = d >> 3;
   const int rs = kThreads / cps;
@@ -592,6 +600,8 @@ __device__ __forceinline__ void compact_slice(uint16_t* kb, uint16_t* vb, int d,
   const int my_ch = chunk0 + tid % cps;
   const int my_off = tid / cps;
   uint16_t* col = my_ch < d8 ? kb + my_ch * 8 : vb + (my_ch - d8) * 8;
+  // fused append: source rows at or above first_stage are staging rows
+  const uint16_t* coln = kn ? (my_ch < d8 ? kn + my_ch * 8 : vn + (my_ch - d8) * 8) : nullptr;
   constexpr int kRingStages = Ring::kStages, kRingItems = Ring::kItems;
   const int tile = rs * kRingItems;
   const int ntiles = r_end > r_begin ? (r_end - r_begin + tile - 1) / tile : 0;
@@ -607,7 +617,9 @@ __device__ __forceinline__ void compact_slice(uint16_t* kb, uint16_t* vb, int d,
         if (on && r < r_end) {
           const int src = perm ? (int)perm[r] : r + 1;
           if (src < n)
-            cp_async16(slot(t % kRingStages, u), col + (size_t)src * d);
+            cp_async16(slot(t % kRingStages, u), src >= first_stage
+                                                     ? coln + (size_t)(src - first_stage) * d
+                                                     : col + (size_t)src * d);
           else
             record_status(status, kStInternal);
         }
@@ -627,6 +639,34 @@ __device__ __forceinline__ void compact_slice(uint16_t* kb, uint16_t* vb, int d,
     issue(t + kRingStages);
   }
   cp_async_wait<0>();
+}
+
+// Fused append of a unit that does not evict: staging rows [0, B) go to
+// cache rows [first, first + B), this CTA's column slice [chunk0, chunk0 +
+// cps) of [K | V].
+__device__ __forceinline__ void copy_new_rows(uint16_t* kb, uint16_t* vb, const uint16_t* kn,
+                                              const uint16_t* vn, int d, int chunk0, int cps,
+                                              int first, int B) {
+  const int d8 = d >> 3;
+  const int items = B * cps;
+  constexpr int U = 4;
+  for (int base = threadIdx.x; base < items; base += kThreads * U) {
+    uint4 q[U];
+    uint16_t* dstp[U];
+#pragma unroll
+    for (int k = 0; k < U; ++k) {
+      const int it = base + k * kThreads;
+      dstp[k] = nullptr;
+      if (it < items) {
+        const int i = it / cps, c = chunk0 + it % cps;
+        q[k] = ld_cg16((c < d8 ? kn + c * 8 : vn + (c - d8) * 8) + (size_t)i * d);
+        dstp[k] = (c < d8 ? kb + c * 8 : vb + (c - d8) * 8) + (size_t)(first + i) * d;
+      }
+    }
+#pragma unroll
+    for (int k = 0; k < U; ++k)
+      if (dstp[k]) st16(dstp[k], q[k]);
+  }
 }
 
 // Hole-fill layout: move h rows, row src_of(i) -> row dst_of(i), of the
@@ -688,17 +728,28 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
   const int u = C > 1 ? (int)cluster_id_x() : (int)blockIdx.x;
   const int d = a.d, d8 = d >> 3;
   const int seq = u / a.units_per_seq;
-  const int n = a.len[seq];
+  const bool fused = a.k_new != nullptr;  // host-checked: ordered block path only
+  const int len0 = a.len[seq];
+  const int n = len0 + (fused ? a.B : 0);
   const int Nb = a.N_dev ? a.N_dev[seq] : a.N;
   const size_t ubase = (size_t)u * a.capacity * d;
   uint16_t* kb = a.k + ubase;
   uint16_t* vb = a.v + ubase;
   const uint16_t* sb = a.score_k ? kb : vb;  // rows the mean and the scores come from
-  auto vrow = [&](int r) -> const uint16_t* { return vb + (size_t)r * d; };
-  auto srow = [&](int r) -> const uint16_t* { return sb + (size_t)r * d; };
+  // fused append: rows at or above first_stage come from the staging buffers
+  const uint16_t* knu = fused ? a.k_new + (size_t)u * a.B * d : nullptr;
+  const uint16_t* vnu = fused ? a.v_new + (size_t)u * a.B * d : nullptr;
+  const uint16_t* snu = a.score_k ? knu : vnu;
+  const int first_stage = fused ? n - a.B : INT_MAX;
+  auto vrow = [&](int r) -> const uint16_t* {
+    return r >= first_stage ? vnu + (size_t)(r - first_stage) * d : vb + (size_t)r * d;
+  };
+  auto srow = [&](int r) -> const uint16_t* {
+    return r >= first_stage ? snu + (size_t)(r - first_stage) * d : sb + (size_t)r * d;
+  };
 
   // ---- validation: uniform across the cluster (per-sequence values only) ---
-  if (n < 0 || n > a.capacity || (a.mu_running && !a.score_only && a.B > n)) {
+  if (len0 < 0 || n > a.capacity || (a.mu_running && !a.score_only && a.B > n)) {
     if (rank == 0 && tid == 0) record_status(a.status, kStDeviceLen);
     return;
   }
@@ -729,6 +780,7 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
   auto pos_of = [&](int r) -> int { return r < first_new ? posu[r] : pnew + (r - first_new); };
 
   if (!evict && !a.score_only) {
+    if (fused) copy_new_rows(kb, vb, knu, vnu, d, chunk0, cps, first_stage, a.B);
     if (hf && rank == 0)
       for (int r = max(first_new, 0) + tid; r < n; r += kThreads) posu[r] = pnew + (r - first_new);
     // ---- nothing to evict: identity outputs, running sum += appended rows ---
@@ -849,13 +901,23 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
         }
       }
     };
-    const uint16_t* rows = sb + (size_t)r0 * d;
     bool fast = false;
     if constexpr (VAR != 1) {  // head dims 64, 128, 256: one 16-byte chunk per lane
+      // cache rows [r0, c_end), then (fused append) staging rows [c_end, r1)
+      const int c_end = min(r1, max(r0, first_stage));
+      auto run = [&](auto lanes) {
+        constexpr int LPR = decltype(lanes)::value;
+        if (c_end > r0)
+          score_rows_fast<VAR, LPR, Ring>(sb + (size_t)r0 * d, c_end - r0, S.mu, finish_row, ring);
+        if (r1 > c_end)
+          score_rows_fast<VAR, LPR, Ring>(
+              snu + (size_t)(c_end - first_stage) * d, r1 - c_end, S.mu,
+              [&](int j, float s) { finish_row(j + (c_end - r0), s); }, ring);
+      };
       fast = true;
-      if (d == 128) score_rows_fast<VAR, 16, Ring>(rows, r1 - r0, S.mu, finish_row, ring);
-      else if (d == 256) score_rows_fast<VAR, 32, Ring>(rows, r1 - r0, S.mu, finish_row, ring);
-      else if (d == 64) score_rows_fast<VAR, 8, Ring>(rows, r1 - r0, S.mu, finish_row, ring);
+      if (d == 128) run(std::integral_constant<int, 16>{});
+      else if (d == 256) run(std::integral_constant<int, 32>{});
+      else if (d == 64) run(std::integral_constant<int, 8>{});
       else fast = false;
     }
     if (!fast) stream_rows<Ring>(
@@ -1047,8 +1109,9 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
 
   // ---- 6. in-place compaction of this CTA's column slice ---------------
   if constexpr (!HF) {
-    compact_slice<Ring>(kb, vb, d, chunk0, cps, e_first, Nb, n, DECODE ? nullptr : perm, a.status,
-                  ring);
+    // fused append: kept staging rows below the budget are written too
+    compact_slice<Ring>(kb, vb, d, chunk0, cps, min(e_first, first_stage), Nb, n,
+                        DECODE ? nullptr : perm, a.status, ring, knu, vnu, first_stage);
   } else {
     // hole-fill: the kept rows at or above N move into the evicted slots
     // below N, in ascending order (movers: the tail of the kept list; holes:

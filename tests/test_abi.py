@@ -98,6 +98,13 @@ def test_scoring_options_rejected_before_launch(lib):
     # the running sum tracks V: the K-side rule recomputes its mean
     assert lib.vd_evict_block_ex(ref, 16, None, 4, 0, 1, 0x80, 1, None, None, None, None,
                                  None) == 3
+    # fused append: both buffers, B >= 1, 16-byte aligned
+    assert lib.vd_append_evict_block(ref, 0x100, 0x200, 0, 16, None, 0, 0, None, None, None,
+                                     None) == 1
+    assert lib.vd_append_evict_block(ref, 0x100, None, 4, 16, None, 0, 0, None, None, None,
+                                     None) == 1
+    assert lib.vd_append_evict_block(ref, 0x108, 0x200, 4, 16, None, 0, 0, None, None, None,
+                                     None) == 2
     # the hole-fill layout needs both position arrays
     assert lib.vd_evict_block_holefill(ref, 16, None, 4, 0, 0, None, 0x40, None, None, None,
                                        None) == 1

@@ -1,0 +1,166 @@
+"""vd_append_evict_block (append and block eviction in one launch) against
+vd_append followed by vd_evict_block: identical kept slots, scores,
+compacted K/V bytes, running sum and lengths.  The two-call path is the one
+the other tests check against the fp64 oracle.  Needs a GB300."""
+from __future__ import annotations
+
+import contextlib
+import os
+
+import pytest
+import torch
+
+import oracle
+import paper_2609_23314_gb300 as vd
+from paper_2609_23314_gb300 import build, workloads as wl
+from vd_gpu import new_cache, units_view
+
+pytestmark = pytest.mark.gpu
+VARS = [oracle.L2, oracle.DIR, oracle.NORM]
+VAR_IDS = ["l2", "dir", "norm"]
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    build.build()
+    vd.load_library()
+    torch.cuda.set_device(0)
+    yield
+    assert vd.vd_get_device_status() == 0
+
+
+@contextlib.contextmanager
+def cluster_size(c):
+    old = os.environ.get("VD_CLUSTER_SIZE")
+    if c is None:
+        os.environ.pop("VD_CLUSTER_SIZE", None)
+    else:
+        os.environ["VD_CLUSTER_SIZE"] = str(c)
+    try:
+        yield
+    finally:
+        if old is None:
+            os.environ.pop("VD_CLUSTER_SIZE", None)
+        else:
+            os.environ["VD_CLUSTER_SIZE"] = old
+
+
+def setup(d, N, B, lens, seed, cap=None, gen="student_t"):
+    cap = cap or N + B
+    cache = new_cache(len(lens), 2, 2, cap, d)
+    st = wl.TokenStream(gen, cache.units, d, device="cuda", seed=seed)
+    wl.fill_rows(st, units_view(cache.k), units_view(cache.v), cap)
+    cache.len.copy_(torch.tensor(lens, dtype=torch.int32))
+    us = cache.unit_shape()
+    k, v = st.next(B)
+    return cache, k.view(us + (B, d)).contiguous(), v.view(us + (B, d)).contiguous()
+
+
+def run_both(cache, k_new, v_new, B, N, var, mu):
+    us = cache.unit_shape()
+    out = []
+    for fused in (False, True):
+        c = vd.Cache(cache.k.clone(), cache.v.clone(), cache.len.clone())
+        rs = None
+        if mu == vd.VD_MU_RUNNING:
+            rs = torch.zeros(us + (cache.head_dim,), dtype=torch.float64, device="cuda")
+            vd.vd_running_sum_init(c, rs)
+        kept = torch.full(us + (N,), -7, dtype=torch.int32, device="cuda")
+        scores = torch.full(us + (cache.capacity,), float("nan"), device="cuda")
+        if fused:
+            vd.vd_append_evict_block(c, k_new, v_new, B, N, None, var, mu, rs, kept, scores)
+        else:
+            vd.vd_append(c, k_new, v_new, B)
+            vd.vd_evict_block(c, N, None, B, var, mu, rs, kept, scores)
+        assert vd.vd_get_device_status() == 0
+        out.append((c, rs, kept, scores))
+    return out
+
+
+def assert_same(a, b):
+    (ca, rsa, ka, sa), (cb, rsb, kb, sb) = a, b
+    assert torch.equal(ca.len, cb.len)
+    assert torch.equal(ka, kb)
+    # scores: bit-identical where written (NaN elsewhere in both)
+    assert torch.equal(sa.view(torch.int32), sb.view(torch.int32))
+    lens = ca.len.cpu().tolist()
+    per_seq = ca.n_layer * ca.n_kv_head
+    ua, ub = units_view(ca.k), units_view(cb.k)
+    va, vb = units_view(ca.v), units_view(cb.v)
+    for u in range(ca.units):
+        n = lens[u // per_seq]
+        assert torch.equal(ua[u, :n].view(torch.int16), ub[u, :n].view(torch.int16)), u
+        assert torch.equal(va[u, :n].view(torch.int16), vb[u, :n].view(torch.int16)), u
+    if rsa is not None:
+        assert torch.equal(rsa, rsb)
+
+
+@pytest.mark.parametrize("var", VARS, ids=VAR_IDS)
+@pytest.mark.parametrize("d", [64, 128, 200, 256])
+@pytest.mark.parametrize("mu", [vd.VD_MU_RECOMPUTE, vd.VD_MU_RUNNING], ids=["recompute", "running"])
+def test_fused_equals_append_then_evict(var, d, mu):
+    N, B = 160, 48
+    # at budget (steady state), partly over (some new rows stay in place),
+    # below budget after the append (no eviction)
+    lens = [N, N - 20, N - B - 5]
+    cache, k_new, v_new = setup(d, N, B, lens, seed=d + 3 * mu + var)
+    for c in (None, 2):
+        if c is not None and (2 * (d // 8)) % c:
+            continue
+        with cluster_size(c):
+            a, b = run_both(cache, k_new, v_new, B, N, var, mu)
+        assert_same(a, b)
+        assert a[0].len.cpu().tolist() == [N, N, N - 5]
+
+
+@pytest.mark.parametrize("cluster", [1, 4, 8])
+def test_fused_prefill_shape_and_repeated_events(cluster):
+    """Block-processing loop at the benchmark's head dim: five events in a
+    row, fused and two-call, stay identical (running mean carried along)."""
+    d, N, B = 256, 512, 64
+    cache, _, _ = setup(d, N, B, [N, N], seed=41, cap=N + B)
+    st = wl.TokenStream("student_t", cache.units, d, device="cuda", seed=42)
+    us = cache.unit_shape()
+    ca = vd.Cache(cache.k.clone(), cache.v.clone(), cache.len.clone())
+    cb = vd.Cache(cache.k.clone(), cache.v.clone(), cache.len.clone())
+    rsa = torch.zeros(us + (d,), dtype=torch.float64, device="cuda")
+    vd.vd_running_sum_init(ca, rsa)
+    rsb = rsa.clone()
+    with cluster_size(cluster):
+        for _ in range(5):
+            k, v = st.next(B)
+            k, v = k.view(us + (B, d)).contiguous(), v.view(us + (B, d)).contiguous()
+            ka = torch.empty(us + (N,), dtype=torch.int32, device="cuda")
+            kb = torch.empty_like(ka)
+            vd.vd_append(ca, k, v, B)
+            vd.vd_evict_block(ca, N, None, B, vd.VD_SCORE_L2, vd.VD_MU_RUNNING, rsa, ka)
+            vd.vd_append_evict_block(cb, k, v, B, N, None, vd.VD_SCORE_L2, vd.VD_MU_RUNNING, rsb, kb)
+            assert vd.vd_get_device_status() == 0
+            assert torch.equal(ka, kb)
+            assert torch.equal(ca.len, cb.len) and int(cb.len[0]) == N
+            assert torch.equal(ca.k[..., :N, :].view(torch.int16), cb.k[..., :N, :].view(torch.int16))
+            assert torch.equal(ca.v[..., :N, :].view(torch.int16), cb.v[..., :N, :].view(torch.int16))
+            assert torch.equal(rsa, rsb)
+
+
+def test_fused_over_capacity_is_reported_and_untouched():
+    d, N, B = 64, 40, 16
+    cache, k_new, v_new = setup(d, N, B, [N, N - 10], seed=5, cap=N + 8)   # N + B > capacity
+    before_k, before_v = cache.k.clone(), cache.v.clone()
+    vd.vd_append_evict_block(cache, k_new, v_new, B, N, None, vd.VD_SCORE_L2, vd.VD_MU_RECOMPUTE)
+    assert vd.vd_get_device_status() == 7      # VD_ERR_DEVICE_LEN (first sequence)
+    assert int(cache.len[0]) == N               # left untouched
+    assert torch.equal(cache.k[0].view(torch.int16), before_k[0].view(torch.int16))
+    assert torch.equal(cache.v[0].view(torch.int16), before_v[0].view(torch.int16))
+    assert int(cache.len[1]) == N               # the other sequence fitted: N - 10 + 16 -> N
+
+
+def test_fused_argument_errors():
+    cache, k_new, v_new = setup(64, 32, 8, [32], seed=1)
+    lib = vd.load_library()
+    call = lambda k, v, B: lib.vd_append_evict_block(  # noqa: E731
+        cache.ref(), k, v, B, 32, None, 0, 0, None, None, None, None)
+    assert call(k_new.data_ptr(), v_new.data_ptr(), 0) == 1          # B < 1
+    assert call(k_new.data_ptr(), None, 8) == 1                      # one buffer missing
+    assert call(k_new.data_ptr() + 2, v_new.data_ptr(), 8) == 2      # not 16-byte aligned
+    assert int(cache.len[0]) == 32
