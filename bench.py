@@ -129,14 +129,17 @@ def kernel_source_hash() -> str:
     return h.hexdigest()[:16]
 
 
-def ncu_traffic(workload: str, layout: str = "ordered"):
+def ncu_traffic(workload: str, layout: str = "ordered", separate: bool = False):
     """DRAM bytes per launch of the eviction kernel from the committed ncu
-    summary, if it was taken on the current kernel sources; else None."""
+    summary, if it was taken on the current kernel sources; else None.
+    separate: an ordered prefill step that appends with vd_append first (its
+    eviction then finds the new rows in the cache, partly still in L2)."""
     path = os.path.join(ROOT, "profiles", "traffic.json")
     try:
         with open(path) as f:
             t = json.load(f)
-        e = t[workload if layout == "ordered" else f"{workload}:{layout}"]
+        key = workload if layout == "ordered" else f"{workload}:{layout}"
+        e = t[key + (":separate" if separate and layout == "ordered" else "")]
         if e.get("source_hash") != kernel_source_hash():
             return None
         return float(e["dram_bytes_per_launch"])
@@ -220,11 +223,14 @@ class Prefill:
     """Block boundary at steady state: append B rows, evict N + B -> N."""
 
     def __init__(self, name, cfg, device, seed, mu, variant, n_blocks=8, layout="ordered",
-                 score_keys=False, weighted=False, dispersion=False):
+                 score_keys=False, weighted=False, dispersion=False, separate_append=False):
         """n_blocks distinct appended blocks are pre-generated and reused in
         order; the benchmark asks for as many as the prompt has (T / B), so
         every timed event appends rows the cache has not seen.  layout
-        "holefill" uses vd_evict_block_holefill with a token-position array."""
+        "holefill" uses vd_evict_block_holefill with a token-position array.
+        The plain ordered step is one vd_append_evict_block call (the new
+        block read straight from its buffer); separate_append, the scoring
+        options and the hole-fill layout append with vd_append first."""
         import torch
         import paper_2609_23314_gb300 as vd
         from paper_2609_23314_gb300 import workloads as wl
@@ -268,6 +274,11 @@ class Prefill:
             self.attn = torch.rand(us + (self.cap,), generator=g, device=device) * 0.9
         # per-unit sigma (Sec. 3.1) of the pre-eviction rows, from the score pass
         self.sigma = torch.empty(us, device=device) if dispersion else None
+        self.fused = not (separate_append or self.holefill or score_keys or weighted
+                          or dispersion)
+        if self.fused:
+            self.launches_per_step = 2     # fused append + evict, len update
+        self.pending = None                # the block the next fused call appends
 
     def head_tokens_per_step(self):
         return self.U * (self.N + self.B)
@@ -280,10 +291,17 @@ class Prefill:
     def append_next(self):
         k, v = self.blocks[self.i % len(self.blocks)]
         self.i += 1
-        self.vd.vd_append(self.cache, k, v, self.B)
+        if self.fused:
+            self.pending = (k, v)          # appended by the eviction call itself
+        else:
+            self.vd.vd_append(self.cache, k, v, self.B)
 
     def evict(self, kept=None, scores=None):
-        if self.holefill:
+        if self.fused:
+            k, v = self.pending
+            self.vd.vd_append_evict_block(self.cache, k, v, self.B, self.N, None, self.variant,
+                                          self.mu, self.rs if self.mu else None, kept, scores)
+        elif self.holefill:
             pn = self.pos_new_all[(self.i - 1) % self.pos_new_all.shape[0]]
             self.vd.vd_evict_block_holefill(self.cache, self.N, self.pos, pn, None, self.B,
                                             self.variant, self.mu, self.rs if self.mu else None,
@@ -351,7 +369,10 @@ class Prefill:
 
     def e2e_compute(self, b):
         self.i += 1
-        self.vd.vd_append(self.cache, self.d_in[b][0], self.d_in[b][1], self.B)
+        if self.fused:
+            self.pending = self.d_in[b]
+        else:
+            self.vd.vd_append(self.cache, self.d_in[b][0], self.d_in[b][1], self.B)
 
     def e2e_evict(self, b):
         self.evict(self.d_out[b])
@@ -543,7 +564,8 @@ def run_e2e(w, steps, device):
     host memory and its result (kept slots, or evicted slots for decode)
     copied back, every step.  Three streams overlap the copies with the
     eviction: copy-in (staging buffer b = step % 2), compute (append from the
-    staging buffer, then evict), copy-out; events keep a staging or result
+    staging buffer and evict, in one call where the step is fused), copy-out;
+    events keep a staging or result
     buffer from being reused before its consumer is done.  Returns the time
     from the first copy-in to the last copy-out (ms)."""
     import torch
@@ -568,9 +590,9 @@ def run_e2e(w, steps, device):
             copied[b].record(h2d)
         comp.wait_event(copied[b])
         w.e2e_compute(b)
-        free[b].record(comp)
         comp.wait_event(out[b])
         w.e2e_evict(b)
+        free[b].record(comp)               # the staging buffer is read up to here
         done[b].record(comp)
         with torch.cuda.stream(d2h):
             d2h.wait_event(done[b])
@@ -769,6 +791,8 @@ def run_vd(args):
         _, cfg = wl.config(name)
         if args.n_seq:
             cfg["n_seq"] = args.n_seq
+        if cfg["kind"] == "prefill" and args.separate_append:
+            opts = dict(opts, separate_append=True)
         w = make_workload(name, device, rank_seed(wl.BASE_SEED + cfg["index"], rank),
                           mu if mu_mode is None else mu_mode, variant, args.n_seq,
                           events=args.warmup + steps, layout=layout, **opts)
@@ -786,7 +810,8 @@ def run_vd(args):
                     "h2d_bytes_per_step": m["bi"], "d2h_bytes_per_step": m["bo"]},
             "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                          "frac": achieved / peak,
-                         "traffic": ncu_traffic(name, layout) if not opts else None,
+                         "traffic": ncu_traffic(name, layout, separate=not getattr(w, "fused", True))
+                         if not (set(opts) - {"separate_append"}) else None,
                          "kernel": f"vd::evict_kernel<{variant}, {str(isinstance(w, Decode)).lower()}, "
                                    f"{str(layout == 'holefill').lower()}>",
                          "algorithmic_bytes_per_launch": alg,
@@ -796,6 +821,8 @@ def run_vd(args):
                          if "measured" in peak_src else peak_src},
             "config": {"workload": name, **{k: cfg[k] for k in cfg if k not in ("index", "kind")},
                        "mu": args.mu, "variant": args.variant, "layout": layout,
+                       "append": ("fused into the eviction (vd_append_evict_block)"
+                                  if getattr(w, "fused", False) else "vd_append, then the eviction"),
                        "l2": f"inputs larger than L2: cache {w.cache.k.numel() * 4 / 2**30:.2f} GiB "
                              "of K+V, touched every step", "storage": "bf16"},
         }
@@ -816,6 +843,15 @@ def run_vd(args):
     if args.secondary not in ("", "none") and args.secondary != args.workload:
         secondary = one(args.secondary, args.secondary_steps, args.layout)
         release(secondary)
+    # the same prefill step with a separate vd_append launch before the
+    # eviction (the two-call form), for comparison with the fused step
+    separate = None
+    if (args.extension_steps > 0 and not args.separate_append and args.layout == "ordered"
+            and wl.config(args.workload)[1]["kind"] == "prefill"):
+        r = one(args.workload, args.extension_steps, "ordered", separate_append=True)
+        separate = {"value": r["value"], "step_ms": r["step_ms"], "kernel_ms": r["kern_ms"],
+                    "roofline_frac": r["roofline"]["frac"], "e2e": r["e2e"]["value"]}
+        release(r)
     # the smallest workload's per-event latency (a few units: launch- and
     # latency-bound, reported in microseconds)
     latency = None
@@ -870,6 +906,8 @@ def run_vd(args):
             line["secondary"] = {k: secondary[k] for k in ("workload", "value", "step_ms", "roofline",
                                                            "e2e", "config")}
             line["secondary"]["clocks"] = secondary["m"]["clocks"]
+        if separate is not None:
+            line["separate_append"] = separate
         if latency is not None:
             line["latency"] = latency
         if holefill:
@@ -948,6 +986,9 @@ def main(argv=None):
                     help="steps of the key-side / weighted / dispersion measurements (0: skip)")
     ap.add_argument("--holefill-steps", type=int, default=50,
                     help="steps of the extra hole-fill-layout measurements (0: skip)")
+    ap.add_argument("--separate-append", action="store_true",
+                    help="prefill steps append with vd_append, then evict (default: one "
+                         "vd_append_evict_block call)")
     ap.add_argument("--mu", choices=["running", "recompute"], default="running")
     ap.add_argument("--variant", choices=["l2", "dir", "norm"], default="l2")
     ap.add_argument("--e2e-steps", type=int, default=50)
