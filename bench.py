@@ -132,14 +132,14 @@ def kernel_source_hash() -> str:
 def ncu_traffic(workload: str, layout: str = "ordered", separate: bool = False):
     """DRAM bytes per launch of the eviction kernel from the committed ncu
     summary, if it was taken on the current kernel sources; else None.
-    separate: an ordered prefill step that appends with vd_append first (its
-    eviction then finds the new rows in the cache, partly still in L2)."""
+    separate: a prefill step that appends with vd_append first (its eviction
+    then finds the new rows in the cache, partly still in L2)."""
     path = os.path.join(ROOT, "profiles", "traffic.json")
     try:
         with open(path) as f:
             t = json.load(f)
         key = workload if layout == "ordered" else f"{workload}:{layout}"
-        e = t[key + (":separate" if separate and layout == "ordered" else "")]
+        e = t[key + (":separate" if separate else "")]
         if e.get("source_hash") != kernel_source_hash():
             return None
         return float(e["dram_bytes_per_launch"])
@@ -228,9 +228,9 @@ class Prefill:
         order; the benchmark asks for as many as the prompt has (T / B), so
         every timed event appends rows the cache has not seen.  layout
         "holefill" uses vd_evict_block_holefill with a token-position array.
-        The plain ordered step is one vd_append_evict_block call (the new
-        block read straight from its buffer); separate_append, the scoring
-        options and the hole-fill layout append with vd_append first."""
+        The step is one vd_append_evict_block call (the new block read
+        straight from its buffer) in either layout; separate_append and the
+        scoring options append with vd_append first."""
         import torch
         import paper_2609_23314_gb300 as vd
         from paper_2609_23314_gb300 import workloads as wl
@@ -274,8 +274,7 @@ class Prefill:
             self.attn = torch.rand(us + (self.cap,), generator=g, device=device) * 0.9
         # per-unit sigma (Sec. 3.1) of the pre-eviction rows, from the score pass
         self.sigma = torch.empty(us, device=device) if dispersion else None
-        self.fused = not (separate_append or self.holefill or score_keys or weighted
-                          or dispersion)
+        self.fused = not (separate_append or score_keys or weighted or dispersion)
         if self.fused:
             self.launches_per_step = 2     # fused append + evict, len update
         self.pending = None                # the block the next fused call appends
@@ -299,8 +298,13 @@ class Prefill:
     def evict(self, kept=None, scores=None):
         if self.fused:
             k, v = self.pending
+            hf = {}
+            if self.holefill:
+                hf = dict(pos=self.pos,
+                          pos_first_new=self.pos_new_all[(self.i - 1) % self.pos_new_all.shape[0]])
             self.vd.vd_append_evict_block(self.cache, k, v, self.B, self.N, None, self.variant,
-                                          self.mu, self.rs if self.mu else None, kept, scores)
+                                          self.mu, self.rs if self.mu else None, kept, scores,
+                                          **hf)
         elif self.holefill:
             pn = self.pos_new_all[(self.i - 1) % self.pos_new_all.shape[0]]
             self.vd.vd_evict_block_holefill(self.cache, self.N, self.pos, pn, None, self.B,

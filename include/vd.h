@@ -131,7 +131,7 @@ vd_status vd_evict_block(const vd_cache* c, int32_t N, const int32_t* N_dev, int
  * scores, compacted K/V bytes in slots [0, new len), running sum and len --
  * but the new rows are read straight from the caller's buffers, and only
  * the ones that survive are written into the cache (appended rows that are
- * evicted at once are never stored).  Ordered layout, block path.
+ * evicted at once are never stored).  Block path, either layout.
  *   k_new, v_new  bf16 device [n_seq][n_layer][n_kv_head][B][head_dim],
  *                 16-byte aligned, read only; B >= 1.
  *   len           on entry the rows already cached (the new ones excluded);
@@ -139,12 +139,17 @@ vd_status vd_evict_block(const vd_cache* c, int32_t N, const int32_t* N_dev, int
  *                 happens.
  *   running_sum   (VD_MU_RUNNING) on entry the sum of rows [0, len), on exit
  *                 the sum of rows [0, new len).
+ *   pos, pos_first_new  both null: ordered layout (vd_evict_block); both
+ *                 given: the hole-fill layout, as vd_append followed by
+ *                 vd_evict_block_holefill (arguments as there, pos_first_new
+ *                 the position of the first new row).
  * Other arguments as in vd_evict_block.  A sequence with len + B > capacity
  * is left untouched and records VD_ERR_DEVICE_LEN.  Slots at or above the new
  * len hold unspecified bytes. */
 vd_status vd_append_evict_block(const vd_cache* c, const void* k_new, const void* v_new,
                                 int32_t B, int32_t N, const int32_t* N_dev, vd_variant var,
-                                vd_mu_mode mu, double* running_sum, int32_t* kept_idx_out,
+                                vd_mu_mode mu, double* running_sum, int32_t* pos,
+                                const int32_t* pos_first_new, int32_t* kept_idx_out,
                                 float* scores_out, vd_stream_t stream);
 
 /* Decode-step eviction (per-token eviction of the abstract and the Sec. 4

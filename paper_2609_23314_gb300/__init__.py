@@ -68,7 +68,7 @@ def load_library() -> ctypes.CDLL:
             cp = ctypes.POINTER(_VdCache)
             lib.vd_score.argtypes = [cp, S, P, P]
             lib.vd_evict_block.argtypes = [cp, I32, P, I32, S, S, P, P, P, P]
-            lib.vd_append_evict_block.argtypes = [cp, P, P, I32, I32, P, S, S, P, P, P, P]
+            lib.vd_append_evict_block.argtypes = [cp, P, P, I32, I32, P, S, S, P, P, P, P, P, P]
             lib.vd_evict_decode.argtypes = [cp, I32, P, S, S, P, P, P, P, P]
             lib.vd_evict_block_holefill.argtypes = [cp, I32, P, I32, S, S, P, P, P, P, P, P]
             lib.vd_evict_decode_holefill.argtypes = [cp, I32, P, S, S, P, P, P, P, P, P, P]
@@ -194,8 +194,9 @@ def vd_evict_block(cache: Cache, N: int, N_dev=None, B: int = 0, variant: int = 
 def vd_append_evict_block(cache: Cache, k_new, v_new, B: int, N: int, N_dev=None,
                           variant: int = VD_SCORE_L2, mu: int = VD_MU_RECOMPUTE,
                           running_sum=None, kept_idx_out=None, scores_out=None,
-                          stream=None) -> None:
-    """vd_append followed by vd_evict_block in one launch; k_new, v_new: bf16
+                          stream=None, pos=None, pos_first_new=None) -> None:
+    """vd_append followed by vd_evict_block (or, with pos and pos_first_new,
+    vd_evict_block_holefill) in one launch; k_new, v_new: bf16
     [n_seq, n_layer, n_kv_head, B, head_dim], read straight from the caller's
     buffers (only surviving rows are written into the cache)."""
     torch = _torch()
@@ -208,10 +209,13 @@ def vd_append_evict_block(cache: Cache, k_new, v_new, B: int, N: int, N_dev=None
         _ptr(running_sum, torch.float64, us + (cache.head_dim,), "running_sum", cache.device),
         _ptr(kept_idx_out, torch.int32, us + (int(N),), "kept_idx_out", cache.device),
         _ptr(scores_out, torch.float32, us + (cache.capacity,), "scores_out", cache.device),
+        _ptr(pos, torch.int32, us + (cache.capacity,), "pos", cache.device),
+        _ptr(pos_first_new, torch.int32, (cache.n_seq,), "pos_first_new", cache.device),
     )
     _check(load_library().vd_append_evict_block(cache.ref(), args[0], args[1], int(B), int(N),
                                                 args[2], int(variant), int(mu), args[3],
-                                                args[4], args[5], _stream(stream)),
+                                                args[6], args[7], args[4], args[5],
+                                                _stream(stream)),
            "vd_append_evict_block")
 
 

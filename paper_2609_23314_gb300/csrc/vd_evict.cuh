@@ -677,7 +677,9 @@ __device__ __forceinline__ void copy_new_rows(uint16_t* kb, uint16_t* vb, const 
 template <class SrcOf, class DstOf>
 __device__ __forceinline__ void move_rows(uint16_t* kb, uint16_t* vb, int d, int chunk0, int cps,
                                           int h, int n, SrcOf src_of, DstOf dst_of,
-                                          unsigned* status) {
+                                          unsigned* status, const uint16_t* kn = nullptr,
+                                          const uint16_t* vn = nullptr,
+                                          int first_stage = INT_MAX) {
   const int d8 = d >> 3;
   const int items = h * cps;
   constexpr int U = 4;
@@ -693,7 +695,10 @@ __device__ __forceinline__ void move_rows(uint16_t* kb, uint16_t* vb, int d, int
         uint16_t* col = c < d8 ? kb + c * 8 : vb + (c - d8) * 8;
         const int sr = src_of(i), dr = dst_of(i);
         if ((unsigned)sr < (unsigned)n && (unsigned)dr < (unsigned)n) {
-          q[k] = ld_cg16(col + (size_t)sr * d);
+          // fused append: sources at or above first_stage are staging rows
+          q[k] = ld_cg16(sr >= first_stage
+                             ? (c < d8 ? kn + c * 8 : vn + (c - d8) * 8) + (size_t)(sr - first_stage) * d
+                             : col + (size_t)sr * d);
           dstp[k] = col + (size_t)dr * d;
         } else {
           record_status(status, kStInternal);
@@ -1133,7 +1138,13 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
     }
     auto src = [&](int i) { return DECODE ? n - 1 : (int)perm[Nb - h + i]; };
     auto dst = [&](int i) { return DECODE ? e_first : (int)perm[Nb + i]; };
-    move_rows(kb, vb, d, chunk0, cps, h, n, src, dst, a.status);
+    if (fused && Nb > first_stage) {
+      // fused append: new rows below the budget stay in their slots (the
+      // evicted ones among them are refilled just below)
+      copy_new_rows(kb, vb, knu, vnu, d, chunk0, cps, first_stage, Nb - first_stage);
+      __syncthreads();
+    }
+    move_rows(kb, vb, d, chunk0, cps, h, n, src, dst, a.status, knu, vnu, first_stage);
     if (rank == 0) {
       for (int r = max(first_new, 0) + tid; r < Nb; r += kThreads) posu[r] = pnew + (r - first_new);
       int32_t* ko = a.kept_out ? a.kept_out + (size_t)u * a.N : nullptr;

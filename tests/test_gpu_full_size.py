@@ -39,6 +39,22 @@ def snapshot(cache, units):
     return bits(units_view(cache.k)[it]), bits(units_view(cache.v)[it])
 
 
+def snapshot_step(w, units):
+    """Pre-eviction rows of the benchmark's next step: the cache's rows and,
+    where the step appends inside the eviction call (vd_append_evict_block),
+    the staged block after them.  Returns (k, v, n)."""
+    k, v = snapshot(w.cache, units)
+    n0 = int(w.cache.len[0])
+    if not getattr(w, "fused", False):
+        return k, v, n0
+    it = torch.tensor(units, device=DEV, dtype=torch.long)
+    pk, pv = w.pending
+    k, v = k.copy(), v.copy()
+    k[:, n0:n0 + w.B] = bits(pk.view(w.U, w.B, w.d)[it])
+    v[:, n0:n0 + w.B] = bits(pv.view(w.U, w.B, w.d)[it])
+    return k, v, n0 + w.B
+
+
 def check_sampled(orc, var, cache, units, pre, n_of, N_of, kept, scores):
     post = snapshot(cache, units)
     U = cache.units
@@ -128,13 +144,15 @@ def test_prefill_wide_steady_state_as_benchmarked(orc, var, mu):
     units = sample_units(w.U, 4, 7 + var)
     kept = torch.empty(w.cache.unit_shape() + (w.N,), dtype=torch.int32, device=DEV)
     scores = torch.empty(w.cache.unit_shape() + (w.cap,), dtype=torch.float32, device=DEV)
+    assert w.fused                      # the benchmark's step: one vd_append_evict_block call
     for step in range(3):
         w.append_next()
-        pre = snapshot(w.cache, units)
+        pk, pv, n = snapshot_step(w, units)
+        assert n == w.N + w.B
         w.evict(kept, scores)
         assert vd.vd_get_device_status() == 0
-        n = w.N + w.B
-        check_sampled(orc, var, w.cache, units, pre, lambda s: n, lambda s: w.N, kept, scores)
+        check_sampled(orc, var, w.cache, units, (pk, pv), lambda s: n, lambda s: w.N, kept,
+                      scores)
     if mu == "running":
         check_running_sum(w.cache, w.rs)
     del w
@@ -265,8 +283,8 @@ def test_holefill_full_size_as_benchmarked(orc, name):
     scores = torch.empty(w.cache.unit_shape() + (cap,), dtype=torch.float32, device=DEV)
     for step in range(4):
         w.append_next()
-        n = int(w.cache.len[0])
-        pre = snapshot(w.cache, units)
+        pk, pv, n = snapshot_step(w, units)
+        pre = (pk, pv)
         pre_pos = w.pos.view(U, cap)[it].cpu().numpy().copy()
         pn = w.pos_new_all[w.i - 1].cpu().numpy()
         for i, u in enumerate(units):

@@ -159,8 +159,86 @@ def test_fused_argument_errors():
     cache, k_new, v_new = setup(64, 32, 8, [32], seed=1)
     lib = vd.load_library()
     call = lambda k, v, B: lib.vd_append_evict_block(  # noqa: E731
-        cache.ref(), k, v, B, 32, None, 0, 0, None, None, None, None)
+        cache.ref(), k, v, B, 32, None, 0, 0, None, None, None, None, None, None)
     assert call(k_new.data_ptr(), v_new.data_ptr(), 0) == 1          # B < 1
     assert call(k_new.data_ptr(), None, 8) == 1                      # one buffer missing
     assert call(k_new.data_ptr() + 2, v_new.data_ptr(), 8) == 2      # not 16-byte aligned
     assert int(cache.len[0]) == 32
+
+
+def run_both_holefill(cache, k_new, v_new, B, N, var, mu, lens):
+    us = cache.unit_shape()
+    cap = cache.capacity
+    out = []
+    for fused in (False, True):
+        c = vd.Cache(cache.k.clone(), cache.v.clone(), cache.len.clone())
+        pos = torch.arange(cap, dtype=torch.int32, device="cuda").repeat(c.units).view(
+            us + (cap,)).contiguous()
+        pos_new = torch.tensor(lens, dtype=torch.int32, device="cuda")  # position of the first new row
+        rs = None
+        if mu == vd.VD_MU_RUNNING:
+            rs = torch.zeros(us + (cache.head_dim,), dtype=torch.float64, device="cuda")
+            vd.vd_running_sum_init(c, rs)
+        kept = torch.full(us + (N,), -7, dtype=torch.int32, device="cuda")
+        scores = torch.full(us + (cap,), float("nan"), device="cuda")
+        if fused:
+            vd.vd_append_evict_block(c, k_new, v_new, B, N, None, var, mu, rs, kept, scores,
+                                     pos=pos, pos_first_new=pos_new)
+        else:
+            vd.vd_append(c, k_new, v_new, B)
+            vd.vd_evict_block_holefill(c, N, pos, pos_new, None, B, var, mu, rs, kept, scores)
+        assert vd.vd_get_device_status() == 0
+        out.append((c, rs, kept, scores, pos))
+    return out
+
+
+@pytest.mark.parametrize("var", VARS, ids=VAR_IDS)
+@pytest.mark.parametrize("mu", [vd.VD_MU_RECOMPUTE, vd.VD_MU_RUNNING], ids=["recompute", "running"])
+@pytest.mark.parametrize("d", [128, 200])
+def test_fused_holefill_equals_append_then_evict(var, mu, d):
+    N, B = 160, 48
+    lens = [N, N - 20, N - B - 5]
+    cache, k_new, v_new = setup(d, N, B, lens, seed=d + 5 * mu + var)
+    for c in (None, 1, 2):
+        with cluster_size(c):
+            a, b = run_both_holefill(cache, k_new, v_new, B, N, var, mu, lens)
+        assert_same(a[:4], b[:4])
+        new_lens = a[0].len.cpu().tolist()
+        assert new_lens == [N, N, N - 5]
+        per_seq = cache.n_layer * cache.n_kv_head
+        pa, pb = a[4].view(cache.units, -1), b[4].view(cache.units, -1)
+        for u in range(cache.units):
+            n = new_lens[u // per_seq]
+            assert torch.equal(pa[u, :n], pb[u, :n]), u
+
+
+def test_fused_holefill_repeated_events():
+    """Five hole-fill block events in a row at the benchmark's head dim, fused
+    and two-call, stay identical (positions and running mean carried along)."""
+    d, N, B = 256, 512, 64
+    cache, _, _ = setup(d, N, B, [N, N], seed=51, cap=N + B)
+    st = wl.TokenStream("student_t", cache.units, d, device="cuda", seed=52)
+    us = cache.unit_shape()
+    cap = N + B
+    ca = vd.Cache(cache.k.clone(), cache.v.clone(), cache.len.clone())
+    cb = vd.Cache(cache.k.clone(), cache.v.clone(), cache.len.clone())
+    pa = torch.arange(cap, dtype=torch.int32, device="cuda").repeat(ca.units).view(us + (cap,)).contiguous()
+    pb = pa.clone()
+    rsa = torch.zeros(us + (d,), dtype=torch.float64, device="cuda")
+    vd.vd_running_sum_init(ca, rsa)
+    rsb = rsa.clone()
+    for e in range(5):
+        k, v = st.next(B)
+        k, v = k.view(us + (B, d)).contiguous(), v.view(us + (B, d)).contiguous()
+        pn = torch.full((cache.n_seq,), N + e * B, dtype=torch.int32, device="cuda")
+        ka = torch.empty(us + (N,), dtype=torch.int32, device="cuda")
+        kb = torch.empty_like(ka)
+        vd.vd_append(ca, k, v, B)
+        vd.vd_evict_block_holefill(ca, N, pa, pn, None, B, vd.VD_SCORE_L2, vd.VD_MU_RUNNING, rsa, ka)
+        vd.vd_append_evict_block(cb, k, v, B, N, None, vd.VD_SCORE_L2, vd.VD_MU_RUNNING, rsb, kb,
+                                 pos=pb, pos_first_new=pn)
+        assert vd.vd_get_device_status() == 0
+        assert torch.equal(ka, kb) and torch.equal(ca.len, cb.len)
+        assert torch.equal(ca.k[..., :N, :].view(torch.int16), cb.k[..., :N, :].view(torch.int16))
+        assert torch.equal(ca.v[..., :N, :].view(torch.int16), cb.v[..., :N, :].view(torch.int16))
+        assert torch.equal(pa[..., :N], pb[..., :N]) and torch.equal(rsa, rsb)
