@@ -401,10 +401,13 @@ class Prefill:
 class Decode:
     """Decode step at steady state: append one token, evict N + 1 -> N."""
 
-    def __init__(self, name, cfg, device, seed, mu, variant, n_tokens=8, layout="ordered"):
+    def __init__(self, name, cfg, device, seed, mu, variant, n_tokens=8, layout="ordered",
+                 separate_append=False):
         """n_tokens distinct appended tokens are pre-generated and reused in
         order (the benchmark asks for the workload's 1024 decode steps).
-        layout "holefill" uses vd_evict_decode_holefill."""
+        layout "holefill" uses the hole-fill layout.  A step is one
+        vd_append_evict_decode call (the token read from its buffer), or with
+        separate_append vd_append then vd_evict_decode(_holefill)."""
         import torch
         import paper_2609_23314_gb300 as vd
         from paper_2609_23314_gb300 import workloads as wl
@@ -431,7 +434,9 @@ class Decode:
         if mu == vd.VD_MU_RUNNING:
             vd.vd_running_sum_init(self.cache, self.rs)
         self.i = 0
-        self.launches_per_step = 4
+        self.fused = not separate_append
+        self.pending = None
+        self.launches_per_step = 2 if self.fused else 4
         self.holefill = layout == "holefill"
         if self.holefill:
             self.pos = torch.arange(self.cap, dtype=torch.int32, device=device).repeat(
@@ -451,10 +456,22 @@ class Decode:
         if k is None:
             k, v = self.tokens[self.i % len(self.tokens)]
         self.i += 1
-        self.vd.vd_append(self.cache, k, v, 1)
+        if self.fused:
+            self.pending = (k, v)          # appended by the eviction call itself
+        else:
+            self.vd.vd_append(self.cache, k, v, 1)
 
     def evict(self, evicted=None, kept=None, scores=None):
-        if self.holefill:
+        if self.fused:
+            k, v = self.pending
+            hf = {}
+            if self.holefill:
+                hf = dict(pos=self.pos,
+                          pos_first_new=self.pos_new_all[(self.i - 1) % self.pos_new_all.shape[0]])
+            self.vd.vd_append_evict_decode(self.cache, k, v, self.N, None, self.variant, self.mu,
+                                           self.rs if self.mu else None, evicted, kept, scores,
+                                           **hf)
+        elif self.holefill:
             pn = self.pos_new_all[(self.i - 1) % self.pos_new_all.shape[0]]
             self.vd.vd_evict_decode_holefill(self.cache, self.N, self.pos, pn, None, self.variant,
                                              self.mu, self.rs if self.mu else None, evicted,
@@ -516,7 +533,10 @@ class Decode:
 
     def e2e_compute(self, b):
         self.i += 1
-        self.vd.vd_append(self.cache, self.d_in[b][0], self.d_in[b][1], 1)
+        if self.fused:
+            self.pending = self.d_in[b]
+        else:
+            self.vd.vd_append(self.cache, self.d_in[b][0], self.d_in[b][1], 1)
 
     def e2e_evict(self, b):
         self.evict(self.d_out[b])
@@ -551,13 +571,13 @@ def make_workload(name, device, seed, mu, variant, n_seq=None, events=8, layout=
         return Prefill(name, cfg, device, seed, mu, variant, n_blocks=pool, layout=layout, **opts)
     if cfg["kind"] == "decode":
         pool = max(8, min(events, cfg["steps"]))
-        return Decode(name, cfg, device, seed, mu, variant, n_tokens=pool, layout=layout)
+        return Decode(name, cfg, device, seed, mu, variant, n_tokens=pool, layout=layout, **opts)
     # ratio budget: its largest event is a decode step at N = 25% of the final length
     cfg = dict(cfg)
     total = cfg["prompt"] + cfg["gen_tokens"]
     cfg["N"] = wl.budget_at(cfg, total)
     pool = max(8, min(events, cfg["gen_tokens"]))
-    return Decode(name, cfg, device, seed, mu, variant, n_tokens=pool, layout=layout)
+    return Decode(name, cfg, device, seed, mu, variant, n_tokens=pool, layout=layout, **opts)
 
 
 # ---------------------------------------------------------------------------
@@ -795,7 +815,7 @@ def run_vd(args):
         _, cfg = wl.config(name)
         if args.n_seq:
             cfg["n_seq"] = args.n_seq
-        if cfg["kind"] == "prefill" and args.separate_append:
+        if args.separate_append:
             opts = dict(opts, separate_append=True)
         w = make_workload(name, device, rank_seed(wl.BASE_SEED + cfg["index"], rank),
                           mu if mu_mode is None else mu_mode, variant, args.n_seq,

@@ -165,6 +165,23 @@ vd_status vd_evict_decode(const vd_cache* c, int32_t N, const int32_t* N_dev, vd
                           vd_mu_mode mu, double* running_sum, int32_t* evicted_out,
                           int32_t* kept_idx_out, float* scores_out, vd_stream_t stream);
 
+/* One decode step in one launch: the same result as vd_append(c, k_new,
+ * v_new, 1) followed by vd_evict_decode (or, with pos and pos_first_new, by
+ * vd_evict_decode_holefill), with the new token read straight from the
+ * caller's buffers and written into the cache only if it survives.
+ *   k_new, v_new  bf16 device [n_seq][n_layer][n_kv_head][1][head_dim],
+ *                 16-byte aligned, read only.
+ *   len           on entry the cached tokens (the new one excluded), on exit
+ *                 min(len + 1, N_s).
+ *   running_sum   (VD_MU_RUNNING) on entry the sum of rows [0, len).
+ * Other arguments as in vd_evict_decode / vd_evict_decode_holefill.  A
+ * sequence with len + 1 > capacity is left untouched (VD_ERR_DEVICE_LEN). */
+vd_status vd_append_evict_decode(const vd_cache* c, const void* k_new, const void* v_new,
+                                 int32_t N, const int32_t* N_dev, vd_variant var, vd_mu_mode mu,
+                                 double* running_sum, int32_t* pos, const int32_t* pos_first_new,
+                                 int32_t* evicted_out, int32_t* kept_idx_out, float* scores_out,
+                                 vd_stream_t stream);
+
 /* Scores with options, no eviction.
  *   score_keys      0: V rows (ValueDiff and its variants, Sec. 3.2); 1: the
  *                   same rules on K rows, with the mean of K (the key-side

@@ -21,7 +21,7 @@ import threading
 __all__ = [
     "VD_SCORE_L2", "VD_SCORE_DIR", "VD_SCORE_NORM", "VD_MU_RECOMPUTE", "VD_MU_RUNNING",
     "VdError", "Cache", "vd_score", "vd_score_ex", "vd_evict_block", "vd_evict_block_ex",
-    "vd_append_evict_block",
+    "vd_append_evict_block", "vd_append_evict_decode",
     "vd_evict_decode",
     "vd_evict_block_holefill", "vd_evict_decode_holefill", "vd_append",
     "vd_running_sum_init", "vd_workspace_size", "vd_status_string", "vd_get_device_status",
@@ -69,6 +69,7 @@ def load_library() -> ctypes.CDLL:
             lib.vd_score.argtypes = [cp, S, P, P]
             lib.vd_evict_block.argtypes = [cp, I32, P, I32, S, S, P, P, P, P]
             lib.vd_append_evict_block.argtypes = [cp, P, P, I32, I32, P, S, S, P, P, P, P, P, P]
+            lib.vd_append_evict_decode.argtypes = [cp, P, P, I32, P, S, S, P, P, P, P, P, P, P]
             lib.vd_evict_decode.argtypes = [cp, I32, P, S, S, P, P, P, P, P]
             lib.vd_evict_block_holefill.argtypes = [cp, I32, P, I32, S, S, P, P, P, P, P, P]
             lib.vd_evict_decode_holefill.argtypes = [cp, I32, P, S, S, P, P, P, P, P, P, P]
@@ -82,7 +83,7 @@ def load_library() -> ctypes.CDLL:
             lib.vd_status_string.restype = ctypes.c_char_p
             lib.vd_get_device_status.argtypes = [P]
             for f in ("vd_score", "vd_score_ex", "vd_evict_block_ex", "vd_evict_block",
-                      "vd_append_evict_block",
+                      "vd_append_evict_block", "vd_append_evict_decode",
                       "vd_evict_decode", "vd_evict_block_holefill",
                       "vd_evict_decode_holefill", "vd_append", "vd_running_sum_init",
                       "vd_get_device_status"):
@@ -217,6 +218,34 @@ def vd_append_evict_block(cache: Cache, k_new, v_new, B: int, N: int, N_dev=None
                                                 args[6], args[7], args[4], args[5],
                                                 _stream(stream)),
            "vd_append_evict_block")
+
+
+def vd_append_evict_decode(cache: Cache, k_new, v_new, N: int, N_dev=None,
+                           variant: int = VD_SCORE_L2, mu: int = VD_MU_RECOMPUTE,
+                           running_sum=None, evicted_out=None, kept_idx_out=None,
+                           scores_out=None, stream=None, pos=None, pos_first_new=None) -> None:
+    """vd_append of one token followed by vd_evict_decode (or, with pos and
+    pos_first_new, vd_evict_decode_holefill) in one launch; k_new, v_new:
+    bf16 [n_seq, n_layer, n_kv_head, 1, head_dim]."""
+    torch = _torch()
+    us = cache.unit_shape()
+    shape = us + (1, cache.head_dim)
+    args = (
+        _ptr(k_new, torch.bfloat16, shape, "k_new", cache.device),
+        _ptr(v_new, torch.bfloat16, shape, "v_new", cache.device),
+        _ptr(N_dev, torch.int32, (cache.n_seq,), "N_dev", cache.device),
+        _ptr(running_sum, torch.float64, us + (cache.head_dim,), "running_sum", cache.device),
+        _ptr(pos, torch.int32, us + (cache.capacity,), "pos", cache.device),
+        _ptr(pos_first_new, torch.int32, (cache.n_seq,), "pos_first_new", cache.device),
+        _ptr(evicted_out, torch.int32, us, "evicted_out", cache.device),
+        _ptr(kept_idx_out, torch.int32, us + (int(N),), "kept_idx_out", cache.device),
+        _ptr(scores_out, torch.float32, us + (cache.capacity,), "scores_out", cache.device),
+    )
+    _check(load_library().vd_append_evict_decode(cache.ref(), args[0], args[1], int(N), args[2],
+                                                 int(variant), int(mu), args[3], args[4],
+                                                 args[5], args[6], args[7], args[8],
+                                                 _stream(stream)),
+           "vd_append_evict_decode")
 
 
 def vd_evict_decode(cache: Cache, N: int, N_dev=None, variant: int = VD_SCORE_L2,

@@ -343,7 +343,7 @@ vd_status run(const vd_cache* c, int32_t N, const int32_t* N_dev, int32_t B, vd_
   if (holefill && (!pos || !pos_new)) return VD_ERR_INVALID_ARG;
   const bool fused = k_new != nullptr || v_new != nullptr;
   if (fused) {
-    if (!k_new || !v_new || B < 1 || decode || score_only) return VD_ERR_INVALID_ARG;
+    if (!k_new || !v_new || B < 1 || score_only) return VD_ERR_INVALID_ARG;
     if ((reinterpret_cast<uintptr_t>(k_new) | reinterpret_cast<uintptr_t>(v_new)) & 15u)
       return VD_ERR_ALIGNMENT;
   }
@@ -419,6 +419,16 @@ vd_status vd_append_evict_block(const vd_cache* c, const void* k_new, const void
   return run(c, N, N_dev, B, var, mu, running_sum, nullptr, kept_idx_out, scores_out,
              reinterpret_cast<cudaStream_t>(stream), false, false, pos, pos_first_new, 0,
              nullptr, nullptr, k_new, v_new);
+}
+
+vd_status vd_append_evict_decode(const vd_cache* c, const void* k_new, const void* v_new,
+                                 int32_t N, const int32_t* N_dev, vd_variant var, vd_mu_mode mu,
+                                 double* running_sum, int32_t* pos, const int32_t* pos_first_new,
+                                 int32_t* evicted_out, int32_t* kept_idx_out, float* scores_out,
+                                 vd_stream_t stream) {
+  return run(c, N, N_dev, 1, var, mu, running_sum, evicted_out, kept_idx_out, scores_out,
+             reinterpret_cast<cudaStream_t>(stream), true, false, pos, pos_first_new, 0, nullptr,
+             nullptr, k_new, v_new);
 }
 
 vd_status vd_evict_block(const vd_cache* c, int32_t N, const int32_t* N_dev, int32_t B,

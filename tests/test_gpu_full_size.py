@@ -179,9 +179,14 @@ def test_decode_batched_1024_steps(orc):
         k, v = st.next(1)
         w.append_next(k.view(us + (1, d)), v.view(us + (1, d)))
         if step in (0, 511, 1023):
-            pre = snapshot(w.cache, units)
+            assert w.fused                  # the benchmark's step: one vd_append_evict_decode call
+            pk, pv, n = snapshot_step(w, units)
+            assert n == N + 1
+            pre = (pk, pv)
             pre_k = units_view(w.cache.k)[sub].clone()
             pre_v = units_view(w.cache.v)[sub].clone()
+            pre_k[:, N] = w.pending[0].view(U, d)[sub]     # the staged token at slot N
+            pre_v[:, N] = w.pending[1].view(U, d)[sub]
             w.evict(evicted, kept, scores)
             assert vd.vd_get_device_status() == 0
             check_sampled(orc, oracle.L2, w.cache, units, pre, lambda s: N + 1, lambda s: N, kept,

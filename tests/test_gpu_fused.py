@@ -242,3 +242,67 @@ def test_fused_holefill_repeated_events():
         assert torch.equal(ca.k[..., :N, :].view(torch.int16), cb.k[..., :N, :].view(torch.int16))
         assert torch.equal(ca.v[..., :N, :].view(torch.int16), cb.v[..., :N, :].view(torch.int16))
         assert torch.equal(pa[..., :N], pb[..., :N]) and torch.equal(rsa, rsb)
+
+
+@pytest.mark.parametrize("var", VARS, ids=VAR_IDS)
+@pytest.mark.parametrize("mu", [vd.VD_MU_RECOMPUTE, vd.VD_MU_RUNNING], ids=["recompute", "running"])
+@pytest.mark.parametrize("layout", ["ordered", "holefill"])
+def test_fused_decode_steps(var, mu, layout):
+    """Twelve decode steps, vd_append_evict_decode against vd_append +
+    vd_evict_decode(_holefill): identical evicted slots, kept slots, scores,
+    cache rows, positions, running sum and lengths; one sequence starts below
+    its budget and grows into it."""
+    d, N = 128, 96
+    lens = [N, N - 3]
+    cache, _, _ = setup(d, N, 1, lens, seed=61 + var + 3 * mu, cap=N + 1, gen="drift")
+    st = wl.TokenStream("drift", cache.units, d, device="cuda", seed=62)
+    us = cache.unit_shape()
+    cap = N + 1
+    hf = layout == "holefill"
+    ca = vd.Cache(cache.k.clone(), cache.v.clone(), cache.len.clone())
+    cb = vd.Cache(cache.k.clone(), cache.v.clone(), cache.len.clone())
+    pa = torch.arange(cap, dtype=torch.int32, device="cuda").repeat(ca.units).view(us + (cap,)).contiguous()
+    pb = pa.clone()
+    rsa = rsb = None
+    if mu == vd.VD_MU_RUNNING:
+        rsa = torch.zeros(us + (d,), dtype=torch.float64, device="cuda")
+        vd.vd_running_sum_init(ca, rsa)
+        rsb = rsa.clone()
+    nextpos = torch.tensor(lens, dtype=torch.int32, device="cuda")
+    for step in range(12):
+        k, v = st.next(1)
+        k, v = k.view(us + (1, d)).contiguous(), v.view(us + (1, d)).contiguous()
+        outs = []
+        for fused in (False, True):
+            c, p, rs = (cb, pb, rsb) if fused else (ca, pa, rsa)
+            ev = torch.full(us, -7, dtype=torch.int32, device="cuda")
+            kept = torch.full(us + (N,), -7, dtype=torch.int32, device="cuda")
+            sc = torch.full(us + (cap,), float("nan"), device="cuda")
+            hfa = dict(pos=p, pos_first_new=nextpos) if hf else {}
+            if fused:
+                vd.vd_append_evict_decode(c, k, v, N, None, var, mu, rs, ev, kept, sc, **hfa)
+            else:
+                vd.vd_append(c, k, v, 1)
+                if hf:
+                    vd.vd_evict_decode_holefill(c, N, p, nextpos, None, var, mu, rs, ev, kept, sc)
+                else:
+                    vd.vd_evict_decode(c, N, None, var, mu, rs, ev, kept, sc)
+            assert vd.vd_get_device_status() == 0
+            outs.append((ev, kept, sc))
+        (ea, ka, sa), (eb, kb, sb) = outs
+        assert torch.equal(ea, eb) and torch.equal(ka, kb)
+        assert torch.equal(sa.view(torch.int32), sb.view(torch.int32))
+        assert torch.equal(ca.len, cb.len)
+        lens_now = ca.len.cpu().tolist()
+        per_seq = ca.n_layer * ca.n_kv_head
+        for u in range(ca.units):
+            n = lens_now[u // per_seq]
+            for x, y in ((ca.k, cb.k), (ca.v, cb.v)):
+                assert torch.equal(units_view(x)[u, :n].view(torch.int16),
+                                   units_view(y)[u, :n].view(torch.int16)), (step, u)
+            if hf:
+                assert torch.equal(pa.view(ca.units, -1)[u, :n], pb.view(ca.units, -1)[u, :n])
+        if rsa is not None:
+            assert torch.equal(rsa, rsb)
+        nextpos += 1
+    assert ca.len.cpu().tolist() == [N, N]
