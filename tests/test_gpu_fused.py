@@ -306,3 +306,47 @@ def test_fused_decode_steps(var, mu, layout):
             assert torch.equal(rsa, rsb)
         nextpos += 1
     assert ca.len.cpu().tolist() == [N, N]
+
+
+def test_fused_per_sequence_budgets():
+    """Per-sequence budgets (N_dev): block and decode steps, fused against the
+    two-call path, including a sequence whose budget lies below its length."""
+    d, N, B = 128, 120, 24
+    lens = [100, 120, 60, 119]
+    Nd = torch.tensor([110, 120, 40, 80], dtype=torch.int32, device="cuda")
+    cache, k_new, v_new = setup(d, N, B, lens, seed=71, cap=N + B)
+    us = cache.unit_shape()
+    res = []
+    for fused in (False, True):
+        c = vd.Cache(cache.k.clone(), cache.v.clone(), cache.len.clone())
+        rs = torch.zeros(us + (d,), dtype=torch.float64, device="cuda")
+        vd.vd_running_sum_init(c, rs)
+        kept = torch.full(us + (N,), -7, dtype=torch.int32, device="cuda")
+        if fused:
+            vd.vd_append_evict_block(c, k_new, v_new, B, N, Nd, vd.VD_SCORE_L2, vd.VD_MU_RUNNING,
+                                     rs, kept)
+        else:
+            vd.vd_append(c, k_new, v_new, B)
+            vd.vd_evict_block(c, N, Nd, B, vd.VD_SCORE_L2, vd.VD_MU_RUNNING, rs, kept)
+        assert vd.vd_get_device_status() == 0
+        # then one decode step with the same budgets
+        st = wl.TokenStream("drift", c.units, d, device="cuda", seed=72)
+        k1, v1 = st.next(1)
+        k1, v1 = k1.view(us + (1, d)).contiguous(), v1.view(us + (1, d)).contiguous()
+        ev = torch.full(us, -7, dtype=torch.int32, device="cuda")
+        if fused:
+            vd.vd_append_evict_decode(c, k1, v1, N, Nd, vd.VD_SCORE_L2, vd.VD_MU_RUNNING, rs, ev)
+        else:
+            vd.vd_append(c, k1, v1, 1)
+            vd.vd_evict_decode(c, N, Nd, vd.VD_SCORE_L2, vd.VD_MU_RUNNING, rs, ev)
+        assert vd.vd_get_device_status() == 0
+        res.append((c, rs, kept, ev))
+    (ca, rsa, ka, ea), (cb, rsb, kb, eb) = res
+    assert torch.equal(ca.len, cb.len) and torch.equal(ka, kb) and torch.equal(ea, eb)
+    assert torch.equal(rsa, rsb)
+    assert ca.len.cpu().tolist() == [110, 120, 40, 80]
+    per_seq = ca.n_layer * ca.n_kv_head
+    for u in range(ca.units):
+        n = ca.len.cpu().tolist()[u // per_seq]
+        assert torch.equal(units_view(ca.k)[u, :n].view(torch.int16), units_view(cb.k)[u, :n].view(torch.int16))
+        assert torch.equal(units_view(ca.v)[u, :n].view(torch.int16), units_view(cb.v)[u, :n].view(torch.int16))
