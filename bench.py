@@ -845,7 +845,9 @@ def run_vd(args):
                          if "measured" in peak_src else peak_src},
             "config": {"workload": name, **{k: cfg[k] for k in cfg if k not in ("index", "kind")},
                        "mu": args.mu, "variant": args.variant, "layout": layout,
-                       "append": ("fused into the eviction (vd_append_evict_block)"
+                       "append": (("fused into the eviction (vd_append_evict_decode)"
+                                   if isinstance(w, Decode) else
+                                   "fused into the eviction (vd_append_evict_block)")
                                   if getattr(w, "fused", False) else "vd_append, then the eviction"),
                        "l2": f"inputs larger than L2: cache {w.cache.k.numel() * 4 / 2**30:.2f} GiB "
                              "of K+V, touched every step", "storage": "bf16"},
