@@ -121,11 +121,18 @@ def hbm_peak():
 
 
 def kernel_source_hash() -> str:
+    """Hash of the CUDA sources' code (comments and white space removed), the
+    key of the committed ncu traffic: a capture stays valid until the code
+    itself changes."""
+    import re
     h = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_2609_23314_gb300", "csrc")
     for name in sorted(os.listdir(csrc)):
-        with open(os.path.join(csrc, name), "rb") as f:
-            h.update(name.encode() + f.read())
+        with open(os.path.join(csrc, name)) as f:
+            text = f.read()
+        text = re.sub(r"/\*.*?\*/", " ", text, flags=re.S)
+        text = re.sub(r"//[^\n]*", " ", text)
+        h.update(name.encode() + " ".join(text.split()).encode())
     return h.hexdigest()[:16]
 
 

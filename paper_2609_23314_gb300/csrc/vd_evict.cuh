@@ -116,9 +116,10 @@ struct EvictArgs {
   int32_t score_k;         // 1: mean and scores from K (key-side rules)
   const float* weights;    // nullable [U][capacity]: attention weights a_j (block path)
   float* disp_out;         // nullable [U]: std of the L2 scores of the scored rows
-  // fused append (ordered block path): the B new rows are read from these
-  // staging buffers ([U][B][d] bf16 each) instead of the cache, len does not
-  // count them yet, and only the kept ones are written (nullable: unfused)
+  // fused append (block or decode, either layout): the B new rows are read
+  // from these staging buffers ([U][B][d] bf16 each) instead of the cache,
+  // len does not count them yet, and only the kept ones are written
+  // (nullable: the rows were appended beforehand)
   const uint16_t* k_new;
   const uint16_t* v_new;
 };
@@ -733,7 +734,7 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
   const int u = C > 1 ? (int)cluster_id_x() : (int)blockIdx.x;
   const int d = a.d, d8 = d >> 3;
   const int seq = u / a.units_per_seq;
-  const bool fused = a.k_new != nullptr;  // host-checked: ordered block path only
+  const bool fused = a.k_new != nullptr;  // the new rows are still in the staging buffers
   const int len0 = a.len[seq];
   const int n = len0 + (fused ? a.B : 0);
   const int Nb = a.N_dev ? a.N_dev[seq] : a.N;
