@@ -54,8 +54,13 @@ typedef enum {
   VD_OK = 0,
   VD_ERR_INVALID_ARG = 1, /* null pointer, non-positive size, N out of range, ... */
   VD_ERR_ALIGNMENT = 2,   /* K/V not 16-byte aligned, or head_dim % 8 != 0 */
-  VD_ERR_UNSUPPORTED = 3, /* shape beyond what the kernels handle (head_dim > 256,
-                             capacity too large for on-chip selection) */
+  VD_ERR_UNSUPPORTED = 3, /* shape beyond what the kernels handle: head_dim > 256;
+                             block eviction with capacity > 65536 (16-bit slot
+                             lists) or whose on-chip keys and slot lists do not
+                             fit one CTA's shared memory at any cluster size
+                             (about 41 KB + capacity * (2 + 4 / C) bytes <= 227 KB,
+                             C <= head_dim / 4): at head_dim >= 64 every
+                             capacity up to 65536 fits */
   VD_ERR_NONFINITE = 4,   /* device: a score was NaN or infinite */
   VD_ERR_TIMEOUT = 5,     /* reserved: no kernel in this library waits on a flag */
   VD_ERR_CUDA = 6,        /* a CUDA runtime call failed (launch error, ...) */

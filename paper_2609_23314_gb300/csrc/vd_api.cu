@@ -231,14 +231,15 @@ bool cluster_allowed(int c, int d) {
 // synchronisation dominates and grows with C): the smallest C with at least
 // 0.85 of a wave.  With none such, the largest allowed C.  (Measured on
 // GB300: prefill_wide ordered C=8 (4.4 waves) 0.574 ms vs C=4 (2.2) 0.586;
-// hole-fill C=2 (1.1 waves) 0.205 vs C=4 0.216; decode C=1.)  want
+// hole-fill C=2 (1.1 waves) 0.205 vs C=4 0.216; decode C=1.)  Where no C
+// with 64-byte segments fits the shared memory (a large capacity at a small
+// head dim), the smallest C that fits.  want
 // (VD_CLUSTER_SIZE: 1, 2, 4, 8 or 16) overrides the choice, for tuning.
 int choose_cluster(const void* kern, long long units, int d, int capacity, bool with_select,
                    bool holefill, int want, const DeviceState& st, size_t* smem_out) {
-  int chosen = 0, fallback = 0, largest = 1;
+  int chosen = 0, fallback = 0, largest = 0, narrow = 0;
   for (int c = 1; c <= 16; c *= 2) {
     if (want >= 1 && c != want) continue;
-    if (want < 1 && !cluster_allowed(c, d)) continue;
     if ((d / 8 * 2) % c) continue;
     const size_t smem = vd::smem_layout(capacity, c, with_select).total;
     if (smem > (size_t)st.smem_optin) continue;
@@ -248,6 +249,12 @@ int choose_cluster(const void* kern, long long units, int d, int capacity, bool 
       continue;
     }
     if (occ < 1 || !cluster_fits(kern, units, c, smem)) continue;
+    if (want < 1 && !cluster_allowed(c, d)) {
+      // narrower row segments than preferred: only when nothing else fits
+      // (a large capacity at a small head dim)
+      if (narrow == 0) narrow = c;
+      continue;
+    }
     largest = c;
     const double waves = (double)(units * c) / ((double)st.sms * occ);
     const bool full_wave = waves >= 0.85 && waves <= 1.0;
@@ -266,7 +273,7 @@ int choose_cluster(const void* kern, long long units, int d, int capacity, bool 
     }
     if (fallback == 0 && (full_wave || waves >= 2.0)) fallback = c;
   }
-  if (chosen == 0) chosen = fallback ? fallback : largest;
+  if (chosen == 0) chosen = fallback ? fallback : largest ? largest : narrow ? narrow : 1;
   *smem_out = vd::smem_layout(capacity, chosen, with_select).total;
   return chosen;
 }
