@@ -260,8 +260,8 @@ class Prefill:
                                 v.view(us + (self.B, self.d)).contiguous()))
         self.mu, self.variant = mu, variant
         self.rs = torch.zeros(us + (self.d,), dtype=torch.float64, device=device)
-        if mu == vd.VD_MU_RUNNING:
-            vd.vd_running_sum_init(self.cache, self.rs)
+        if mu == vd.VD_MU_RUNNING:   # the running sum of the scored tensor (K for the key side)
+            vd.vd_running_sum_init_ex(self.cache, score_keys, self.rs)
         self.kept = None
         self.i = 0
         self.launches_per_step = 4     # append + len add, evict + len clamp
@@ -904,13 +904,13 @@ def run_vd(args):
             r = one(name, args.holefill_steps, "holefill")
             release(r)
             holefill[name] = {k: r[k] for k in ("value", "step_ms", "roofline", "e2e")}
-    # scoring options on the primary (prefill) workload: the K-side rule (mean
-    # recomputed from K: K is read twice), attention weights, and the
+    # scoring options on the primary (prefill) workload: the K-side rule (with
+    # the running mean of K, as the primary's of V), attention weights, and the
     # per-unit dispersion sigma_V from a score-only pass, and as a by-product
     # of the eviction's own score pass
     extensions = {}
     if args.extension_steps > 0 and wl.config(args.workload)[1]["kind"] == "prefill":
-        for key, opts, mu_mode in (("key_side", dict(score_keys=True), vd.VD_MU_RECOMPUTE),
+        for key, opts, mu_mode in (("key_side", dict(score_keys=True), None),
                                    ("attention_weighted", dict(weighted=True), None),
                                    ("dispersion_by_product", dict(dispersion=True), None)):
             r = one(args.workload, args.extension_steps, "ordered", mu_mode, **opts)

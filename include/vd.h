@@ -202,9 +202,10 @@ vd_status vd_score_ex(const vd_cache* c, vd_variant var, int32_t score_keys, flo
                       float* dispersion_out, vd_stream_t stream);
 
 /* vd_evict_block with scoring options:
- *   score_keys  1: select on the K-side rule (mean of K); only with
- *               VD_MU_RECOMPUTE (the running sum tracks V) -> else
- *               VD_ERR_UNSUPPORTED.  K and V are still both compacted.
+ *   score_keys  1: select on the K-side rule (mean of K).  With
+ *               VD_MU_RUNNING, running_sum holds sums of K rows (seed it with
+ *               vd_running_sum_init_ex(c, 1, ...)).  K and V are still both
+ *               compacted.
  *   attn        nullable fp32 device [..][capacity]: an attention weight a_j
  *               in [0, 1) per cached token; the score becomes
  *               a_j / (1 - a_j) * s_j, the FastCAOTE form of App. A
@@ -269,6 +270,12 @@ vd_status vd_append(const vd_cache* c, const void* k_new, const void* v_new, int
 /* running_sum[u][:] = sum of V rows [0, len) of unit u, from scratch (fp64
  * [n_seq][n_layer][n_kv_head][head_dim], device). */
 vd_status vd_running_sum_init(const vd_cache* c, double* running_sum, vd_stream_t stream);
+
+/* vd_running_sum_init for the tensor a running mean tracks: of_keys = 0 the V
+ * rows (ValueDiff and its variants), 1 the K rows (the key-side rules of
+ * vd_evict_block_ex with score_keys = 1).  Same layout and errors. */
+vd_status vd_running_sum_init_ex(const vd_cache* c, int32_t of_keys, double* running_sum,
+                                 vd_stream_t stream);
 
 /* Device scratch the calls need beyond their arguments: always 0 (the fused
  * kernels keep every intermediate on chip). */

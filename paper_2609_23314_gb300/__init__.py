@@ -24,7 +24,8 @@ __all__ = [
     "vd_append_evict_block", "vd_append_evict_decode",
     "vd_evict_decode",
     "vd_evict_block_holefill", "vd_evict_decode_holefill", "vd_append",
-    "vd_running_sum_init", "vd_workspace_size", "vd_status_string", "vd_get_device_status",
+    "vd_running_sum_init", "vd_running_sum_init_ex", "vd_workspace_size", "vd_status_string",
+    "vd_get_device_status",
     "library_path", "load_library",
 ]
 
@@ -77,6 +78,7 @@ def load_library() -> ctypes.CDLL:
             lib.vd_evict_block_ex.argtypes = [cp, I32, P, I32, S, S, P, I32, P, P, P, P, P]
             lib.vd_append.argtypes = [cp, P, P, I32, P]
             lib.vd_running_sum_init.argtypes = [cp, P, P]
+            lib.vd_running_sum_init_ex.argtypes = [cp, I32, P, P]
             lib.vd_workspace_size.argtypes = [cp]
             lib.vd_workspace_size.restype = ctypes.c_size_t
             lib.vd_status_string.argtypes = [S]
@@ -86,6 +88,7 @@ def load_library() -> ctypes.CDLL:
                       "vd_append_evict_block", "vd_append_evict_decode",
                       "vd_evict_decode", "vd_evict_block_holefill",
                       "vd_evict_decode_holefill", "vd_append", "vd_running_sum_init",
+                      "vd_running_sum_init_ex",
                       "vd_get_device_status"):
                 getattr(lib, f).restype = S
             _lib = lib
@@ -351,6 +354,15 @@ def vd_append(cache: Cache, k_new, v_new, B: int, stream=None) -> None:
     kp = _ptr(k_new, torch.bfloat16, shape, "k_new", cache.device)
     vp = _ptr(v_new, torch.bfloat16, shape, "v_new", cache.device)
     _check(load_library().vd_append(cache.ref(), kp, vp, int(B), _stream(stream)), "vd_append")
+
+
+def vd_running_sum_init_ex(cache: Cache, of_keys: bool, running_sum, stream=None) -> None:
+    """fp64 column sums of the cached K rows (of_keys) or V rows, per unit."""
+    torch = _torch()
+    rp = _ptr(running_sum, torch.float64, cache.unit_shape() + (cache.head_dim,), "running_sum",
+              cache.device)
+    _check(load_library().vd_running_sum_init_ex(cache.ref(), int(bool(of_keys)), rp,
+                                                 _stream(stream)), "vd_running_sum_init_ex")
 
 
 def vd_running_sum_init(cache: Cache, running_sum, stream=None) -> None:

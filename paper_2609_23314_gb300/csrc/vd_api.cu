@@ -345,7 +345,6 @@ vd_status run(const vd_cache* c, int32_t N, const int32_t* N_dev, int32_t B, vd_
   }
   if (disp_out && (decode || var != VD_SCORE_L2)) return VD_ERR_INVALID_ARG;
   if (weights && (score_only || decode)) return VD_ERR_INVALID_ARG;
-  if (score_k && mu == VD_MU_RUNNING && !score_only) return VD_ERR_UNSUPPORTED;
   const bool holefill = pos != nullptr || pos_new != nullptr;
   if (holefill && (!pos || !pos_new)) return VD_ERR_INVALID_ARG;
   const bool fused = k_new != nullptr || v_new != nullptr;
@@ -513,6 +512,11 @@ vd_status vd_append(const vd_cache* c, const void* k_new, const void* v_new, int
 }
 
 vd_status vd_running_sum_init(const vd_cache* c, double* running_sum, vd_stream_t stream) {
+  return vd_running_sum_init_ex(c, 0, running_sum, stream);
+}
+
+vd_status vd_running_sum_init_ex(const vd_cache* c, int32_t of_keys, double* running_sum,
+                                 vd_stream_t stream) {
   vd_status r = validate_cache(c);
   if (r != VD_OK) return r;
   if (!running_sum) return VD_ERR_INVALID_ARG;
@@ -522,7 +526,8 @@ vd_status vd_running_sum_init(const vd_cache* c, double* running_sum, vd_stream_
   const long long units = (long long)c->n_seq * c->n_layer * c->n_kv_head;
   const size_t smem = vd::smem_layout(c->capacity, 1, false).total;
   vd_rsum_init_kernel<<<(unsigned)units, kThreads, smem, reinterpret_cast<cudaStream_t>(stream)>>>(
-      static_cast<const uint16_t*>(c->v), c->len, running_sum, c->n_layer * c->n_kv_head,
+      static_cast<const uint16_t*>(of_keys ? c->k : c->v), c->len, running_sum,
+      c->n_layer * c->n_kv_head,
       c->capacity, c->head_dim, lanes_per_row(c->head_dim), st->status);
   if (cudaGetLastError() != cudaSuccess) return VD_ERR_CUDA;
   return VD_OK;

@@ -743,13 +743,11 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
   uint16_t* vb = a.v + ubase;
   const uint16_t* sb = a.score_k ? kb : vb;  // rows the mean and the scores come from
   // fused append: rows at or above first_stage come from the staging buffers
+  // (srow: a row of the scored tensor, V or K)
   const uint16_t* knu = fused ? a.k_new + (size_t)u * a.B * d : nullptr;
   const uint16_t* vnu = fused ? a.v_new + (size_t)u * a.B * d : nullptr;
   const uint16_t* snu = a.score_k ? knu : vnu;
   const int first_stage = fused ? n - a.B : INT_MAX;
-  auto vrow = [&](int r) -> const uint16_t* {
-    return r >= first_stage ? vnu + (size_t)(r - first_stage) * d : vb + (size_t)r * d;
-  };
   auto srow = [&](int r) -> const uint16_t* {
     return r >= first_stage ? snu + (size_t)(r - first_stage) * d : sb + (size_t)r * d;
   };
@@ -770,13 +768,16 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
   }
   if (a.score_only && n == 0) return;
 
-  // column slice of [K | V] this CTA compacts and keeps the running sum of
+  // column slice of [K | V] this CTA compacts; the running sum is kept for
+  // the part of it that lies in the scored tensor (V, or K for the key-side
+  // rule): its chunks [tchunk0, tchunk0 + tchunks) of that tensor
   const int cps = (2 * d8) / C;
   const int chunk0 = (int)rank * cps;
-  const int vchunk0 = max(chunk0, d8) - d8;
-  const int vchunks = max(0, chunk0 + cps - max(chunk0, d8));
-  int vp = 1;
-  while (vp < vchunks) vp <<= 1;
+  const int tchunk0 = a.score_k ? min(chunk0, d8) : max(chunk0, d8) - d8;
+  const int tchunks = a.score_k ? max(0, min(chunk0 + cps, d8) - chunk0)
+                                : max(0, chunk0 + cps - max(chunk0, d8));
+  int tp = 1;
+  while (tp < tchunks) tp <<= 1;
   const int first_new = n - a.B;
   // hole-fill layout: token positions (rows at or above first_new are the
   // appended ones, numbered from pos_new)
@@ -794,11 +795,11 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
       for (int i = (int)rank * kThreads + tid; i < a.N; i += C * kThreads)
         a.kept_out[(size_t)u * a.N + i] = i < n ? i : -1;
     if (DECODE && a.evicted_out && rank == 0 && tid == 0) a.evicted_out[u] = -1;
-    if (a.mu_running && a.B > 0 && vchunks > 0) {
-      sum_rows<Ring>(vchunk0, vchunks, vp, a.B, [&](int i) { return vrow(first_new + i); },
+    if (a.mu_running && a.B > 0 && tchunks > 0) {
+      sum_rows<Ring>(tchunk0, tchunks, tp, a.B, [&](int i) { return srow(first_new + i); },
                [](int) { return 1.f; }, S, ring);
-      if (tid < vchunks * 8) {
-        const int c = vchunk0 * 8 + tid;
+      if (tid < tchunks * 8) {
+        const int c = tchunk0 * 8 + tid;
         double* sp = a.running_sum + (size_t)u * d + c;
         *sp = *sp + (double)S.acc_hi[c] + (double)S.acc_lo[c];
       }
@@ -1091,22 +1092,22 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
   }
   if (DECODE && a.evicted_out && rank == 0 && tid == 0) a.evicted_out[u] = e_first;
 
-  // ---- 5. running sum: S += appended rows - evicted rows (own V columns) --
-  // The appended rows were already summed for the mean (all but Norm); only
-  // the evicted rows are read again.
-  if (a.mu_running && vchunks > 0) {
+  // ---- 5. running sum: S += appended rows - evicted rows (own columns of
+  // the scored tensor).  The appended rows were already summed for the mean
+  // (all but Norm); only the evicted rows are read again.
+  if (a.mu_running && tchunks > 0) {
     const int B = VAR != 2 ? 0 : a.B;
-    sum_rows<Ring>(vchunk0, vchunks, vp, B + (n - Nb),
+    sum_rows<Ring>(tchunk0, tchunks, tp, B + (n - Nb),
              [&](int i) {
                const int r =
                    i < B ? first_new + i : (DECODE ? e_first : (int)perm[Nb + (i - B)]);
-               if ((unsigned)r < (unsigned)n) return vrow(r);
+               if ((unsigned)r < (unsigned)n) return srow(r);
                record_status(a.status, kStInternal);  // self-check: never expected
-               return vrow(0);
+               return srow(0);
              },
              [&](int i) { return i < B ? 1.f : -1.f; }, S, ring);
-    if (tid < vchunks * 8) {
-      const int c = vchunk0 * 8 + tid;
+    if (tid < tchunks * 8) {
+      const int c = tchunk0 * 8 + tid;
       double* sp = a.running_sum + (size_t)u * d + c;
       const double added = VAR != 2 ? S.snew[c] : 0.0;
       *sp = *sp + added + (double)S.acc_hi[c] + (double)S.acc_lo[c];

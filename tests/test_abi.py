@@ -95,9 +95,10 @@ def test_scoring_options_rejected_before_launch(lib):
                                  None) == 1
     assert lib.vd_score_ex(ref, 2, 0, None, sigma, None) == 1
     assert lib.vd_score_ex(ref, 0, 0, None, None, None) == 1                  # no output
-    # the running sum tracks V: the K-side rule recomputes its mean
-    assert lib.vd_evict_block_ex(ref, 16, None, 4, 0, 1, 0x80, 1, None, None, None, None,
-                                 None) == 3
+    # the running mean needs its sum, for either tensor
+    assert lib.vd_evict_block_ex(ref, 16, None, 4, 0, 1, None, 1, None, None, None, None,
+                                 None) == 1
+    assert lib.vd_running_sum_init_ex(ref, 1, None, None) == 1
     # fused append: both buffers, B >= 1, 16-byte aligned
     assert lib.vd_append_evict_block(ref, 0x100, 0x200, 0, 16, None, 0, 0, None, None, None,
                                      None, None, None) == 1

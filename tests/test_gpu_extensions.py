@@ -200,12 +200,48 @@ def test_dispersion_by_product_running_mean(orc, cluster, monkeypatch):
         assert abs(got[u] - want) <= 1e-5 * want + 1e-6, (u, got[u], want)
 
 
+@pytest.mark.parametrize("var", VARS, ids=VAR_IDS)
+@pytest.mark.parametrize("cluster", [1, 4])
+def test_key_side_running_mean(orc, var, cluster, monkeypatch):
+    """The key-side rule with the running mean: a running sum of K rows (seeded
+    by vd_running_sum_init_ex) carried over block events; each event matches
+    the oracle on K, and the sum stays the K rows' sum."""
+    global _ORC
+    _ORC = orc
+    monkeypatch.setenv("VD_CLUSTER_SIZE", str(cluster))
+    d, N, B = 128, 300, 64
+    cache = filled(2, 2, 2, N + B, d, [N, N - 30], seed=91 + cluster)
+    us = cache.unit_shape()
+    rs = torch.zeros(us + (d,), dtype=torch.float64, device="cuda")
+    vd.vd_running_sum_init_ex(cache, True, rs)
+    st = wl.TokenStream("gauss_outlier", cache.units, d, device="cuda", seed=92)
+    per_seq = cache.n_layer * cache.n_kv_head
+    for event in range(3):
+        k, v = st.next(B)
+        vd.vd_append(cache, k.view(us + (B, d)), v.view(us + (B, d)), B)
+        lens = cache.len.cpu().numpy().copy()
+        pre_k, pre_v = bits(units_view(cache.k)), bits(units_view(cache.v))
+        kept = torch.full(us + (N,), -7, dtype=torch.int32, device="cuda")
+        scores = torch.full(us + (N + B,), float("nan"), device="cuda")
+        vd.vd_evict_block_ex(cache, N, None, B, var, vd.VD_MU_RUNNING, rs, True, None, kept,
+                             scores)
+        assert vd.vd_get_device_status() == 0
+        post_k, post_v = bits(units_view(cache.k)), bits(units_view(cache.v))
+        kh, sh = kept.view(cache.units, N).cpu().numpy(), scores.view(cache.units, -1).cpu().numpy()
+        for u in range(cache.units):
+            n = int(lens[u // per_seq])
+            s_ora = orc.scores(pre_k[u, :n], var)
+            tol = score_tolerance(var, s_ora, pre_k[u, :n], orc.mean(pre_k[u, :n]))
+            check_scored_event(s_ora, tol, pre_k[u], pre_v[u], post_k[u], post_v[u], n, N,
+                               kh[u], sh[u])
+        ref = torch.zeros_like(rs)
+        vd.vd_running_sum_init_ex(cache, True, ref)
+        scale = units_view(cache.k).float().abs().sum(dim=1).max().item()
+        assert torch.max(torch.abs(ref - rs)).item() <= 1e-12 * scale
+
+
 def test_option_errors():
     cache = filled(1, 1, 1, 64, 64, [64], seed=1)
-    rs = torch.zeros(1, 1, 1, 64, dtype=torch.float64, device="cuda")
-    with pytest.raises(vd.VdError) as e:
-        vd.vd_evict_block_ex(cache, 32, None, 0, vd.VD_SCORE_L2, vd.VD_MU_RUNNING, rs, True)
-    assert e.value.code == 3                  # the running sum tracks V only
     with pytest.raises(vd.VdError) as e:
         vd.vd_score_ex(cache, vd.VD_SCORE_DIR, False, None,
                        torch.zeros(1, 1, 1, device="cuda"))
