@@ -591,9 +591,7 @@ template <class Ring>
 __device__ __forceinline__ void compact_slice(uint16_t* kb, uint16_t* vb, int d, int chunk0,
                                               int cps, int r_begin, int r_end, int n,
                                               const uint16_t* perm, unsigned* status,
-                                              uint32_t ring, const uint16_t* kn = nullptr,
-                                              const uint16_t* vn = nullptr,
-                                              int first_stage = INT_MAX) {
+                                              uint32_t ring) {
   const int tid = threadIdx.x;
   const int d8 = d >> 3;
   const int rs = kThreads / cps;
@@ -601,8 +599,6 @@ __device__ __forceinline__ void compact_slice(uint16_t* kb, uint16_t* vb, int d,
   const int my_ch = chunk0 + tid % cps;
   const int my_off = tid / cps;
   uint16_t* col = my_ch < d8 ? kb + my_ch * 8 : vb + (my_ch - d8) * 8;
-  // fused append: source rows at or above first_stage are staging rows
-  const uint16_t* coln = kn ? (my_ch < d8 ? kn + my_ch * 8 : vn + (my_ch - d8) * 8) : nullptr;
   constexpr int kRingStages = Ring::kStages, kRingItems = Ring::kItems;
   const int tile = rs * kRingItems;
   const int ntiles = r_end > r_begin ? (r_end - r_begin + tile - 1) / tile : 0;
@@ -618,9 +614,7 @@ __device__ __forceinline__ void compact_slice(uint16_t* kb, uint16_t* vb, int d,
         if (on && r < r_end) {
           const int src = perm ? (int)perm[r] : r + 1;
           if (src < n)
-            cp_async16(slot(t % kRingStages, u), src >= first_stage
-                                                     ? coln + (size_t)(src - first_stage) * d
-                                                     : col + (size_t)src * d);
+            cp_async16(slot(t % kRingStages, u), col + (size_t)src * d);
           else
             record_status(status, kStInternal);
         }
@@ -667,6 +661,29 @@ __device__ __forceinline__ void copy_new_rows(uint16_t* kb, uint16_t* vb, const 
 #pragma unroll
     for (int k = 0; k < U; ++k)
       if (dstp[k]) st16(dstp[k], q[k]);
+  }
+}
+
+// Fused append, ordered layout: cache rows [r_lo, r_hi) of this CTA's column
+// slice take staging row stage_of(r) (kept new rows; their slots follow
+// every slot fed from the cache, because kept slots are ascending).  A
+// staging index outside [0, B) (never expected) is skipped and recorded.
+template <class StageOf>
+__device__ __forceinline__ void copy_staged_rows(uint16_t* kb, uint16_t* vb, const uint16_t* kn,
+                                                 const uint16_t* vn, int d, int chunk0, int cps,
+                                                 int r_lo, int r_hi, int B, StageOf stage_of,
+                                                 unsigned* status) {
+  const int d8 = d >> 3;
+  const int items = (r_hi - r_lo) * cps;
+  for (int it = threadIdx.x; it < items; it += kThreads) {
+    const int r = r_lo + it / cps, c = chunk0 + it % cps;
+    const int i = stage_of(r);
+    if ((unsigned)i >= (unsigned)B) {
+      record_status(status, kStInternal);
+      continue;
+    }
+    const uint4 q = ld_cg16((c < d8 ? kn + c * 8 : vn + (c - d8) * 8) + (size_t)i * d);
+    st16((c < d8 ? kb + c * 8 : vb + (c - d8) * 8) + (size_t)r * d, q);
   }
 }
 
@@ -751,6 +768,13 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
   auto srow = [&](int r) -> const uint16_t* {
     return r >= first_stage ? snu + (size_t)(r - first_stage) * d : sb + (size_t)r * d;
   };
+  // the start of a range [r, r + m) of rows that lies on one side of
+  // first_stage (nullptr when it straddles it: then srow per row)
+  auto srange = [&](int r, int m) -> const uint16_t* {
+    if (r + m <= first_stage) return sb + (size_t)r * d;
+    if (r >= first_stage) return snu + (size_t)(r - first_stage) * d;
+    return nullptr;
+  };
 
   // ---- validation: uniform across the cluster (per-sequence values only) ---
   if (len0 < 0 || n > a.capacity || (a.mu_running && !a.score_only && a.B > n)) {
@@ -796,7 +820,8 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
         a.kept_out[(size_t)u * a.N + i] = i < n ? i : -1;
     if (DECODE && a.evicted_out && rank == 0 && tid == 0) a.evicted_out[u] = -1;
     if (a.mu_running && a.B > 0 && tchunks > 0) {
-      sum_rows<Ring>(tchunk0, tchunks, tp, a.B, [&](int i) { return srow(first_new + i); },
+      const uint16_t* nb = srange(first_new, a.B);  // the new rows lie on one side
+      sum_rows<Ring>(tchunk0, tchunks, tp, a.B, [&](int i) { return nb + (size_t)i * d; },
                [](int) { return 1.f; }, S, ring);
       if (tid < tchunks * 8) {
         const int c = tchunk0 * 8 + tid;
@@ -822,7 +847,10 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
       p0 = r0;
       p1 = r1;
     }
-    sum_rows<Ring>(0, d8, lpr, max(0, p1 - p0), [&](int i) { return srow(p0 + i); },
+    const int cnt = max(0, p1 - p0);
+    const uint16_t* pb = srange(p0, cnt);  // nullptr only where the range straddles
+    sum_rows<Ring>(0, d8, lpr, cnt,
+                   [&](int i) { return pb ? pb + (size_t)i * d : srow(p0 + i); },
                    [](int) { return 1.f; }, S, ring);
     if (C > 1) cluster_sync(); else __syncthreads();
     if (tid < d) {
@@ -927,8 +955,9 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
       else if (d == 64) run(std::integral_constant<int, 8>{});
       else fast = false;
     }
+    const uint16_t* rb = srange(r0, r1 - r0);  // nullptr only where the range straddles
     if (!fast) stream_rows<Ring>(
-        0, d8, lpr, r1 - r0, [&](int i) { return srow(r0 + i); },
+        0, d8, lpr, r1 - r0, [&](int i) { return rb ? rb + (size_t)i * d : srow(r0 + i); },
         [&](int item, bool in, const uint4& q) {
           float x[8];
           unpack8(q, x);
@@ -1116,9 +1145,33 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
 
   // ---- 6. in-place compaction of this CTA's column slice ---------------
   if constexpr (!HF) {
-    // fused append: kept staging rows below the budget are written too
-    compact_slice<Ring>(kb, vb, d, chunk0, cps, min(e_first, first_stage), Nb, n,
-                        DECODE ? nullptr : perm, a.status, ring, knu, vnu, first_stage);
+    // fused append: kept new rows below the budget are written too.  Their
+    // sources are the staging rows, and they occupy the suffix [r_star, Nb)
+    // of the compaction range (kept slots ascend); the cache-fed part runs
+    // first, then (after a barrier: it may still read rows of that suffix)
+    // the staged rows are copied in.
+    auto src_of = [&](int r) { return DECODE ? r + 1 : (int)perm[r]; };
+    const int r_begin = min(e_first, first_stage);
+    int r_star = Nb;
+    if (fused) {
+      if (tid == 0) {
+        int lo = r_begin, hi = Nb;
+        while (lo < hi) {
+          const int mid = (lo + hi) >> 1;
+          if (src_of(mid) < first_stage) lo = mid + 1; else hi = mid;
+        }
+        S.holes = lo;
+      }
+      __syncthreads();
+      r_star = S.holes;
+    }
+    compact_slice<Ring>(kb, vb, d, chunk0, cps, r_begin, r_star, n, DECODE ? nullptr : perm,
+                        a.status, ring);
+    if (fused && r_star < Nb) {
+      __syncthreads();
+      copy_staged_rows(kb, vb, knu, vnu, d, chunk0, cps, r_star, Nb, a.B,
+                       [&](int r) { return src_of(r) - first_stage; }, a.status);
+    }
   } else {
     // hole-fill: the kept rows at or above N move into the evicted slots
     // below N, in ascending order (movers: the tail of the kept list; holes:
