@@ -16,9 +16,9 @@
 #include "vd_evict.cuh"
 
 namespace vd {
-const void* evict_kernel_l2(bool decode, bool holefill);
-const void* evict_kernel_dir(bool decode, bool holefill);
-const void* evict_kernel_norm(bool decode, bool holefill);
+const void* evict_kernel_l2(bool decode, bool holefill, bool fused);
+const void* evict_kernel_dir(bool decode, bool holefill, bool fused);
+const void* evict_kernel_norm(bool decode, bool holefill, bool fused);
 }  // namespace vd
 
 using vd::kThreads;
@@ -129,11 +129,11 @@ constexpr int kMaxDevices = 64;
 std::mutex g_mu;
 DeviceState g_dev[kMaxDevices];
 
-const void* evict_kernel(vd_variant var, bool decode, bool holefill) {
+const void* evict_kernel(vd_variant var, bool decode, bool holefill, bool fused) {
   switch (var) {
-    case VD_SCORE_L2: return vd::evict_kernel_l2(decode, holefill);
-    case VD_SCORE_DIR: return vd::evict_kernel_dir(decode, holefill);
-    default: return vd::evict_kernel_norm(decode, holefill);
+    case VD_SCORE_L2: return vd::evict_kernel_l2(decode, holefill, fused);
+    case VD_SCORE_DIR: return vd::evict_kernel_dir(decode, holefill, fused);
+    default: return vd::evict_kernel_norm(decode, holefill, fused);
   }
 }
 
@@ -162,8 +162,9 @@ vd_status device_state(DeviceState** out) {
                              st.smem_optin) != cudaSuccess)
       return VD_ERR_CUDA;
     for (int var = 0; var < 3; ++var)
-      for (int kind = 0; kind < 4; ++kind) {
-        const void* kern = evict_kernel((vd_variant)var, (kind & 1) != 0, (kind & 2) != 0);
+      for (int kind = 0; kind < 8; ++kind) {
+        const void* kern =
+            evict_kernel((vd_variant)var, (kind & 1) != 0, (kind & 2) != 0, (kind & 4) != 0);
         if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  st.smem_optin) != cudaSuccess ||
             cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) !=
@@ -362,7 +363,7 @@ vd_status run(const vd_cache* c, int32_t N, const int32_t* N_dev, int32_t B, vd_
   if (!small && c->capacity > 65536) return VD_ERR_UNSUPPORTED;  // 16-bit slot lists
   if (vd::smem_layout(c->capacity, 16, !small).total > (size_t)st->smem_optin)
     return VD_ERR_UNSUPPORTED;
-  const void* kern = evict_kernel(var, small, holefill);
+  const void* kern = evict_kernel(var, small, holefill, fused);
   const long long units = (long long)c->n_seq * c->n_layer * c->n_kv_head;
 
   vd::EvictArgs a;

@@ -731,8 +731,10 @@ __device__ __forceinline__ void move_rows(uint16_t* kb, uint16_t* vb, int d, int
 
 // VAR: 0 L2, 1 Dir, 2 Norm.  DECODE: one-token eviction (arg-min) instead of
 // the radix select.  HF: hole-fill layout (compiled separately, so the ordered
-// layout carries none of its code).
-template <int VAR, bool DECODE, bool HF>
+// layout carries none of its code).  FUSED: the new rows are read from the
+// caller's staging buffers (vd_append_evict_*); the other kernels carry none
+// of that code.
+template <int VAR, bool DECODE, bool HF, bool FUSED>
 __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLOCK_MIN_CTAS)
     evict_kernel(const EvictArgs a) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
@@ -751,7 +753,7 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
   const int u = C > 1 ? (int)cluster_id_x() : (int)blockIdx.x;
   const int d = a.d, d8 = d >> 3;
   const int seq = u / a.units_per_seq;
-  const bool fused = a.k_new != nullptr;  // the new rows are still in the staging buffers
+  constexpr bool fused = FUSED;  // the new rows are still in the staging buffers
   const int len0 = a.len[seq];
   const int n = len0 + (fused ? a.B : 0);
   const int Nb = a.N_dev ? a.N_dev[seq] : a.N;
@@ -850,7 +852,10 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
     const int cnt = max(0, p1 - p0);
     const uint16_t* pb = srange(p0, cnt);  // nullptr only where the range straddles
     sum_rows<Ring>(0, d8, lpr, cnt,
-                   [&](int i) { return pb ? pb + (size_t)i * d : srow(p0 + i); },
+                   [&](int i) -> const uint16_t* {
+                     if constexpr (FUSED) return pb ? pb + (size_t)i * d : srow(p0 + i);
+                     else return pb + (size_t)i * d;
+                   },
                    [](int) { return 1.f; }, S, ring);
     if (C > 1) cluster_sync(); else __syncthreads();
     if (tid < d) {
@@ -957,7 +962,11 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
     }
     const uint16_t* rb = srange(r0, r1 - r0);  // nullptr only where the range straddles
     if (!fast) stream_rows<Ring>(
-        0, d8, lpr, r1 - r0, [&](int i) { return rb ? rb + (size_t)i * d : srow(r0 + i); },
+        0, d8, lpr, r1 - r0,
+        [&](int i) -> const uint16_t* {
+          if constexpr (FUSED) return rb ? rb + (size_t)i * d : srow(r0 + i);
+          else return rb + (size_t)i * d;
+        },
         [&](int item, bool in, const uint4& q) {
           float x[8];
           unpack8(q, x);

@@ -3,11 +3,16 @@
 #include "vd_evict.cuh"
 
 namespace vd {
-const void* evict_kernel_l2(bool decode, bool holefill) {
-  if (holefill)
-    return decode ? reinterpret_cast<const void*>(&evict_kernel<0, true, true>)
-                  : reinterpret_cast<const void*>(&evict_kernel<0, false, true>);
-  return decode ? reinterpret_cast<const void*>(&evict_kernel<0, true, false>)
-                : reinterpret_cast<const void*>(&evict_kernel<0, false, false>);
+const void* evict_kernel_l2(bool decode, bool holefill, bool fused) {
+  const void* k[2][2][2] = {
+      {{reinterpret_cast<const void*>(&evict_kernel<0, false, false, false>),
+        reinterpret_cast<const void*>(&evict_kernel<0, false, false, true>)},
+       {reinterpret_cast<const void*>(&evict_kernel<0, false, true, false>),
+        reinterpret_cast<const void*>(&evict_kernel<0, false, true, true>)}},
+      {{reinterpret_cast<const void*>(&evict_kernel<0, true, false, false>),
+        reinterpret_cast<const void*>(&evict_kernel<0, true, false, true>)},
+       {reinterpret_cast<const void*>(&evict_kernel<0, true, true, false>),
+        reinterpret_cast<const void*>(&evict_kernel<0, true, true, true>)}}};
+  return k[decode][holefill][fused];
 }
 }  // namespace vd

@@ -3,11 +3,16 @@
 #include "vd_evict.cuh"
 
 namespace vd {
-const void* evict_kernel_norm(bool decode, bool holefill) {
-  if (holefill)
-    return decode ? reinterpret_cast<const void*>(&evict_kernel<2, true, true>)
-                  : reinterpret_cast<const void*>(&evict_kernel<2, false, true>);
-  return decode ? reinterpret_cast<const void*>(&evict_kernel<2, true, false>)
-                : reinterpret_cast<const void*>(&evict_kernel<2, false, false>);
+const void* evict_kernel_norm(bool decode, bool holefill, bool fused) {
+  const void* k[2][2][2] = {
+      {{reinterpret_cast<const void*>(&evict_kernel<2, false, false, false>),
+        reinterpret_cast<const void*>(&evict_kernel<2, false, false, true>)},
+       {reinterpret_cast<const void*>(&evict_kernel<2, false, true, false>),
+        reinterpret_cast<const void*>(&evict_kernel<2, false, true, true>)}},
+      {{reinterpret_cast<const void*>(&evict_kernel<2, true, false, false>),
+        reinterpret_cast<const void*>(&evict_kernel<2, true, false, true>)},
+       {reinterpret_cast<const void*>(&evict_kernel<2, true, true, false>),
+        reinterpret_cast<const void*>(&evict_kernel<2, true, true, true>)}}};
+  return k[decode][holefill][fused];
 }
 }  // namespace vd
