@@ -736,7 +736,7 @@ def measure_dispersion(args, device, variant, peak, rank):
     achieved = alg / (ms / 1e3) / 1e9
     res = {"value": w.U * n / (ms / 1e3), "step_ms": ms,
            "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
-                        "frac": achieved / peak, "kernel": "vd::evict_kernel<0, true, false> (score only)",
+                        "frac": achieved / peak, "kernel": "vd::evict_kernel<0, true, false, false> (score only)",
                         "algorithmic_bytes_per_launch": alg, "kernel_ms": ms,
                         "sigma_v_mean": float(sigma.mean().item()),
                         "sigma_k_mean": float(sigma_k.mean().item()),
@@ -844,7 +844,8 @@ def run_vd(args):
                          "traffic": ncu_traffic(name, layout, separate=not getattr(w, "fused", True))
                          if not (set(opts) - {"separate_append"}) else None,
                          "kernel": f"vd::evict_kernel<{variant}, {str(isinstance(w, Decode)).lower()}, "
-                                   f"{str(layout == 'holefill').lower()}>",
+                                   f"{str(layout == 'holefill').lower()}, "
+                                   f"{str(getattr(w, 'fused', False)).lower()}>",
                          "algorithmic_bytes_per_launch": alg,
                          "nominal_bytes_per_launch": nominal,
                          "moved_rows_per_launch": m["moved"],

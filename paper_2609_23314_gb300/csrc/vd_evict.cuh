@@ -675,15 +675,28 @@ __device__ __forceinline__ void copy_staged_rows(uint16_t* kb, uint16_t* vb, con
                                                  unsigned* status) {
   const int d8 = d >> 3;
   const int items = (r_hi - r_lo) * cps;
-  for (int it = threadIdx.x; it < items; it += kThreads) {
-    const int r = r_lo + it / cps, c = chunk0 + it % cps;
-    const int i = stage_of(r);
-    if ((unsigned)i >= (unsigned)B) {
-      record_status(status, kStInternal);
-      continue;
+  constexpr int U = 4;  // loads in flight per thread before the stores
+  for (int base = threadIdx.x; base < items; base += kThreads * U) {
+    uint4 q[U];
+    uint16_t* dstp[U];
+#pragma unroll
+    for (int k = 0; k < U; ++k) {
+      const int it = base + k * kThreads;
+      dstp[k] = nullptr;
+      if (it < items) {
+        const int r = r_lo + it / cps, c = chunk0 + it % cps;
+        const int i = stage_of(r);
+        if ((unsigned)i < (unsigned)B) {
+          q[k] = ld_cg16((c < d8 ? kn + c * 8 : vn + (c - d8) * 8) + (size_t)i * d);
+          dstp[k] = (c < d8 ? kb + c * 8 : vb + (c - d8) * 8) + (size_t)r * d;
+        } else {
+          record_status(status, kStInternal);
+        }
+      }
     }
-    const uint4 q = ld_cg16((c < d8 ? kn + c * 8 : vn + (c - d8) * 8) + (size_t)i * d);
-    st16((c < d8 ? kb + c * 8 : vb + (c - d8) * 8) + (size_t)r * d, q);
+#pragma unroll
+    for (int k = 0; k < U; ++k)
+      if (dstp[k]) st16(dstp[k], q[k]);
   }
 }
 
