@@ -197,8 +197,15 @@ vd_status vd_append_evict_decode(const vd_cache* c, const void* k_new, const voi
  *                   standard deviation over its len tokens of the L2 distance
  *                   from the mean -- sigma_V (or sigma_K with score_keys) of
  *                   Sec. 3.1 (population std).  Requires var == VD_SCORE_L2.
- * At least one of the two outputs must be given.  The mean is recomputed. */
-vd_status vd_score_ex(const vd_cache* c, vd_variant var, int32_t score_keys, float* scores_out,
+ *   mu, running_sum  VD_MU_RECOMPUTE: the mean is summed from the len rows
+ *                   (every row is read twice).  VD_MU_RUNNING: the mean is
+ *                   running_sum / len (fp64 [n_seq][n_layer][n_kv_head]
+ *                   [head_dim], read only: the sums of the len rows of the
+ *                   scored tensor that the eviction calls maintain), so the
+ *                   rows are read once.  running_sum must be non-null then.
+ * At least one of the two outputs must be given. */
+vd_status vd_score_ex(const vd_cache* c, vd_variant var, vd_mu_mode mu,
+                      const double* running_sum, int32_t score_keys, float* scores_out,
                       float* dispersion_out, vd_stream_t stream);
 
 /* vd_evict_block with scoring options:

@@ -74,7 +74,7 @@ def load_library() -> ctypes.CDLL:
             lib.vd_evict_decode.argtypes = [cp, I32, P, S, S, P, P, P, P, P]
             lib.vd_evict_block_holefill.argtypes = [cp, I32, P, I32, S, S, P, P, P, P, P, P]
             lib.vd_evict_decode_holefill.argtypes = [cp, I32, P, S, S, P, P, P, P, P, P, P]
-            lib.vd_score_ex.argtypes = [cp, S, I32, P, P, P]
+            lib.vd_score_ex.argtypes = [cp, S, S, P, I32, P, P, P]
             lib.vd_evict_block_ex.argtypes = [cp, I32, P, I32, S, S, P, I32, P, P, P, P, P]
             lib.vd_append.argtypes = [cp, P, P, I32, P]
             lib.vd_running_sum_init.argtypes = [cp, P, P]
@@ -269,14 +269,19 @@ def vd_evict_decode(cache: Cache, N: int, N_dev=None, variant: int = VD_SCORE_L2
 
 
 def vd_score_ex(cache: Cache, variant: int, score_keys: bool = False, scores_out=None,
-                dispersion_out=None, stream=None) -> None:
-    """Scores of V (or K) rows and/or the per-unit dispersion sigma."""
+                dispersion_out=None, stream=None, mu: int = VD_MU_RECOMPUTE,
+                running_sum=None) -> None:
+    """Scores of V (or K) rows and/or the per-unit dispersion sigma; with
+    mu=VD_MU_RUNNING the mean is running_sum / len (fp64 [n_seq, n_layer,
+    n_kv_head, head_dim], read only), so the rows are read once."""
     torch = _torch()
     us = cache.unit_shape()
     sc = _ptr(scores_out, torch.float32, us + (cache.capacity,), "scores_out", cache.device)
     dp = _ptr(dispersion_out, torch.float32, us, "dispersion_out", cache.device)
-    _check(load_library().vd_score_ex(cache.ref(), int(variant), int(bool(score_keys)), sc, dp,
-                                      _stream(stream)), "vd_score_ex")
+    rs = _ptr(running_sum, torch.float64, us + (cache.head_dim,), "running_sum", cache.device)
+    _check(load_library().vd_score_ex(cache.ref(), int(variant), int(mu), rs,
+                                      int(bool(score_keys)), sc, dp, _stream(stream)),
+           "vd_score_ex")
 
 
 def vd_evict_block_ex(cache: Cache, N: int, N_dev=None, B: int = 0, variant: int = VD_SCORE_L2,

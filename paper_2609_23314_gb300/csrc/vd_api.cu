@@ -382,7 +382,7 @@ vd_status run(const vd_cache* c, int32_t N, const int32_t* N_dev, int32_t B, vd_
   a.capacity = c->capacity;
   a.N = score_only ? 1 : N;
   a.B = decode ? 1 : B;
-  a.mu_running = (!score_only && mu == VD_MU_RUNNING) ? 1 : 0;
+  a.mu_running = mu == VD_MU_RUNNING ? 1 : 0;
   a.score_only = score_only ? 1 : 0;
   a.pos = pos;
   a.pos_new = pos_new;
@@ -452,11 +452,14 @@ vd_status vd_evict_decode(const vd_cache* c, int32_t N, const int32_t* N_dev, vd
              reinterpret_cast<cudaStream_t>(stream), true, false);
 }
 
-vd_status vd_score_ex(const vd_cache* c, vd_variant var, int32_t score_keys, float* scores_out,
+vd_status vd_score_ex(const vd_cache* c, vd_variant var, vd_mu_mode mu,
+                      const double* running_sum, int32_t score_keys, float* scores_out,
                       float* dispersion_out, vd_stream_t stream) {
-  return run(c, 1, nullptr, 0, var, VD_MU_RECOMPUTE, nullptr, nullptr, nullptr, scores_out,
-             reinterpret_cast<cudaStream_t>(stream), false, true, nullptr, nullptr, score_keys,
-             nullptr, dispersion_out);
+  if (mu == VD_MU_RUNNING && !running_sum) return VD_ERR_INVALID_ARG;
+  // the score-only kernel reads the running sum and never writes it
+  return run(c, 1, nullptr, 0, var, mu, const_cast<double*>(running_sum), nullptr, nullptr,
+             scores_out, reinterpret_cast<cudaStream_t>(stream), false, true, nullptr, nullptr,
+             score_keys, nullptr, dispersion_out);
 }
 
 vd_status vd_evict_block_ex(const vd_cache* c, int32_t N, const int32_t* N_dev, int32_t B,

@@ -108,7 +108,7 @@ struct EvictArgs {
   int32_t N;              // scalar budget, kept_out stride, N_dev bound
   int32_t B;              // rows appended since the previous eviction
   int32_t mu_running;     // 1: mean from running_sum + appended rows
-  int32_t score_only;     // 1: vd_score (mean recomputed, no eviction)
+  int32_t score_only;     // 1: vd_score / vd_score_ex (no eviction)
   int32_t cluster;        // C, CTAs per unit
   int32_t* pos;            // hole-fill layout: token positions [U][capacity]
   const int32_t* pos_new;  // hole-fill layout: position of row len - B, [n_seq]
@@ -852,7 +852,8 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
   const int r0 = min(n, (int)rank * rows_per), r1 = min(n, r0 + rows_per);
   const int lpr = a.lpr;
   if (VAR != 2) {
-    const bool run = a.mu_running && !a.score_only;
+    // running mean: S plus the appended rows (none for score-only calls)
+    const bool run = a.mu_running;
     int p0, p1;
     if (run) {  // the appended rows, spread over the cluster
       const int per = (a.B + C - 1) / C;

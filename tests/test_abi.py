@@ -93,8 +93,10 @@ def test_scoring_options_rejected_before_launch(lib):
     # sigma is defined on the L2 distance
     assert lib.vd_evict_block_ex(ref, 16, None, 4, 1, 0, None, 0, None, None, None, sigma,
                                  None) == 1
-    assert lib.vd_score_ex(ref, 2, 0, None, sigma, None) == 1
-    assert lib.vd_score_ex(ref, 0, 0, None, None, None) == 1                  # no output
+    assert lib.vd_score_ex(ref, 2, 0, None, 0, None, sigma, None) == 1
+    assert lib.vd_score_ex(ref, 0, 0, None, 0, None, None, None) == 1        # no output
+    assert lib.vd_score_ex(ref, 0, 1, None, 0, None, sigma, None) == 1       # running, no sum
+    assert lib.vd_score_ex(ref, 0, 5, None, 0, None, sigma, None) == 1       # unknown mean mode
     # the running mean needs its sum, for either tensor
     assert lib.vd_evict_block_ex(ref, 16, None, 4, 0, 1, None, 1, None, None, None, None,
                                  None) == 1

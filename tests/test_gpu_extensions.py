@@ -144,6 +144,49 @@ def test_dispersion_matches_oracle(orc, keys, cluster, monkeypatch):
         assert abs(got[u] - want) <= 1e-5 * want + 1e-6, (u, got[u], want)
 
 
+@pytest.mark.parametrize("keys", [False, True], ids=["v", "k"])
+@pytest.mark.parametrize("var", VARS, ids=VAR_IDS)
+@pytest.mark.parametrize("cluster", [1, 2, 4])
+def test_score_ex_running_mean(orc, keys, var, cluster, monkeypatch):
+    """vd_score_ex with the mean taken from a running sum (the rows read
+    once): scores (and sigma, for L2) match the oracle on the current rows,
+    both right after the sum is seeded and after an eviction carried it; the
+    sum is only read; rows at or above len are not written."""
+    monkeypatch.setenv("VD_CLUSTER_SIZE", str(cluster))
+    d, N, B = 128, 300, 64
+    cache = filled(3, 2, 2, N + B, d, [N, N - 40, 1], seed=71 + cluster, gen="student_t")
+    us = cache.unit_shape()
+    per_seq = cache.n_layer * cache.n_kv_head
+    rs = torch.zeros(us + (d,), dtype=torch.float64, device="cuda")
+    vd.vd_running_sum_init_ex(cache, keys, rs)
+    st = wl.TokenStream("gauss_outlier", cache.units, d, device="cuda", seed=72)
+    for stage in range(2):
+        if stage == 1:  # one block event with the running mean carries the sum
+            k, v = st.next(B)
+            vd.vd_append(cache, k.view(us + (B, d)), v.view(us + (B, d)), B)
+            vd.vd_evict_block_ex(cache, N, None, B, var, vd.VD_MU_RUNNING, rs, keys)
+        lens = cache.len.cpu().numpy().copy()
+        rs_before = rs.clone()
+        sc = torch.full(us + (N + B,), float("nan"), device="cuda")
+        sig = torch.full(us, -1.0, device="cuda") if var == oracle.L2 else None
+        vd.vd_score_ex(cache, var, keys, sc, sig, mu=vd.VD_MU_RUNNING, running_sum=rs)
+        assert vd.vd_get_device_status() == 0
+        assert torch.equal(rs, rs_before)
+        src = bits(units_view(cache.k if keys else cache.v))
+        sh = sc.view(cache.units, -1).cpu().numpy()
+        for u in range(cache.units):
+            n = int(lens[u // per_seq])
+            s_ora = orc.scores(src[u, :n], var)
+            tol = score_tolerance(var, s_ora, src[u, :n], orc.mean(src[u, :n]))
+            err = np.abs(sh[u, :n].astype(np.float64) - s_ora)
+            assert np.all(err <= tol), (stage, u, float(err.max()))
+            assert np.all(np.isnan(sh[u, n:]))
+            if sig is not None:
+                want = orc.dispersion(src[u, :n])
+                got = float(sig.view(-1)[u].item())
+                assert abs(got - want) <= 1e-5 * want + 1e-6, (stage, u, got, want)
+
+
 @pytest.mark.parametrize("keys", [False, True], ids=["sigma_v", "sigma_k"])
 @pytest.mark.parametrize("cluster", [1, 2, 4])
 @pytest.mark.parametrize("weighted", [False, True], ids=["plain", "weighted"])
@@ -246,6 +289,10 @@ def test_option_errors():
         vd.vd_score_ex(cache, vd.VD_SCORE_DIR, False, None,
                        torch.zeros(1, 1, 1, device="cuda"))
     assert e.value.code == 1                  # sigma is defined on L2 distances
+    with pytest.raises(vd.VdError) as e:
+        vd.vd_score_ex(cache, vd.VD_SCORE_L2, False, torch.zeros(1, 1, 1, 64, device="cuda"),
+                       mu=vd.VD_MU_RUNNING)
+    assert e.value.code == 1                  # a running mean needs its sum
     with pytest.raises(vd.VdError) as e:
         vd.vd_evict_block_ex(cache, 32, variant=vd.VD_SCORE_NORM,
                              dispersion_out=torch.zeros(1, 1, 1, device="cuda"))
