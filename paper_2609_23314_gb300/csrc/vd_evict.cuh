@@ -132,7 +132,7 @@ struct Smem {
   float muhat[256];
   float acc_hi[256];  // this CTA's partial column sums (read by peer CTAs)
   float acc_lo[256];
-  double snew[256];       // running mode: sum of the appended rows, per column
+  double snew[256];       // running mode: the running sum plus the appended rows
   uint32_t hist[2][256];  // this CTA's radix histograms (read by peers)
   uint32_t ghist[256];
   int scan[kWarps];
@@ -864,6 +864,8 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
       p1 = r1;
     }
     const int cnt = max(0, p1 - p0);
+    // the running sum is loaded before the row sum, whose latency hides it
+    const double rs_own = run && tid < d ? a.running_sum[(size_t)u * d + tid] : 0.0;
     const uint16_t* pb = srange(p0, cnt);  // nullptr only where the range straddles
     sum_rows<Ring>(0, d8, lpr, cnt,
                    [&](int i) -> const uint16_t* {
@@ -886,8 +888,8 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
       }
       double sum = (double)t.hi + (double)t.lo;
       if (run) {
-        S.snew[tid] = sum;
-        sum += a.running_sum[(size_t)u * d + tid];
+        sum += rs_own;
+        S.snew[tid] = sum;  // phase 5 starts from it
       }
       S.mu[tid] = (float)(sum / (double)n);
     }
@@ -1146,9 +1148,15 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
 
   // ---- 5. running sum: S += appended rows - evicted rows (own columns of
   // the scored tensor).  The appended rows were already summed for the mean
-  // (all but Norm); only the evicted rows are read again.
+  // (all but Norm: S plus them is in S.snew); only the evicted rows are read
+  // again.  Norm loads S before the row sum, whose latency hides it.
   if (a.mu_running && tchunks > 0) {
     const int B = VAR != 2 ? 0 : a.B;
+    double base = 0.0;
+    if (tid < tchunks * 8) {
+      const int c = tchunk0 * 8 + tid;
+      base = VAR != 2 ? S.snew[c] : a.running_sum[(size_t)u * d + c] + 0.0;
+    }
     sum_rows<Ring>(tchunk0, tchunks, tp, B + (n - Nb),
              [&](int i) {
                const int r =
@@ -1160,9 +1168,7 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
              [&](int i) { return i < B ? 1.f : -1.f; }, S, ring);
     if (tid < tchunks * 8) {
       const int c = tchunk0 * 8 + tid;
-      double* sp = a.running_sum + (size_t)u * d + c;
-      const double added = VAR != 2 ? S.snew[c] : 0.0;
-      *sp = *sp + added + (double)S.acc_hi[c] + (double)S.acc_lo[c];
+      a.running_sum[(size_t)u * d + c] = base + (double)S.acc_hi[c] + (double)S.acc_lo[c];
     }
   }
 
