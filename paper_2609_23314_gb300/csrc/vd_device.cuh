@@ -165,12 +165,17 @@ __device__ __forceinline__ unsigned cluster_id_x() {
   return r;
 }
 
+// Not the .aligned forms: an .aligned barrier must be executed by all threads
+// of a warp together, and several call sites follow code in which a warp's
+// threads diverged (a loop with a per-thread trip count, a tid == 0 branch).
+// The compiler gives an inline-asm barrier no reconvergence point, so with
+// .aligned, whether a warp arrives converged would depend on code layout.
 __device__ __forceinline__ void cluster_arrive() {
-  asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory");
+  asm volatile("barrier.cluster.arrive.release;" ::: "memory");
 }
 
 __device__ __forceinline__ void cluster_wait() {
-  asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory");
+  asm volatile("barrier.cluster.wait.acquire;" ::: "memory");
 }
 
 __device__ __forceinline__ void cluster_sync() {
