@@ -1,0 +1,140 @@
+"""Seeded random sweep of the fused entry points against the fp64 oracle.
+
+Each case draws a shape (sequences, layers, KV heads, a head dim that is a
+multiple of 8 up to 256), a budget N, a block size B (1 for decode), ragged
+lengths at or below N, a scoring rule, a mean mode, a layout and a cluster
+size, per-sequence budgets or not, fills the cache from the workload
+generators, and runs two events through vd_append_evict_block /
+vd_append_evict_decode (or, in some cases, the two-call form: vd_append,
+then the eviction of that layout).  Every unit of every
+event is checked like the rest of the parity suite: scores within 1e-5
+relative of the oracle's (plus the fp32 rounding floor), the kept set of
+Eq. (eviction) outside near ties, the compacted K and V rows bit for bit, the
+new length, and the running sum against a from-scratch sum.  Needs a GB300.
+"""
+from __future__ import annotations
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import paper_2609_23314_gb300 as vd
+from paper_2609_23314_gb300 import build, workloads as wl
+from test_gpu_holefill import check_holefill_event
+from vd_gpu import bits, check_event, new_cache, units_view
+
+pytestmark = pytest.mark.gpu
+HEAD_DIMS = [8, 16, 24, 40, 64, 72, 128, 136, 200, 256]
+N_CASES = 48
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    build.build()
+    vd.load_library()
+    torch.cuda.set_device(0)
+    yield
+    assert vd.vd_get_device_status() == 0
+
+
+def draw_case(i):
+    r = np.random.default_rng(7919 * (i + 1))
+    d = int(r.choice(HEAD_DIMS))
+    decode = bool(r.random() < 0.35)
+    N = int(r.integers(1, 401))
+    B = 1 if decode else int(r.integers(1, 97))
+    n_seq, L, H = int(r.integers(1, 4)), int(r.integers(1, 3)), int(r.integers(1, 4))
+    budgets = [int(r.integers(1, N + 1)) for _ in range(n_seq)] if r.random() < 0.3 else None
+    lens = [int(r.integers(max(0, Nb - 3 * B), Nb + 1))
+            for Nb in (budgets if budgets else [N] * n_seq)]
+    allowed = [c for c in (1, 2, 4, 8, 16) if (2 * (d // 8)) % c == 0]
+    return dict(d=d, decode=decode, N=N, B=B, n_seq=n_seq, L=L, H=H, lens=lens,
+                budgets=budgets, two_call=bool(r.random() < 0.2),
+                cap=N + B + int(r.integers(0, 17)),
+                var=int(r.integers(0, 3)), mu=int(r.integers(0, 2)),
+                holefill=bool(r.random() < 0.4),
+                cluster=int(r.choice(allowed)) if r.random() < 0.5 else 0,
+                gen=str(r.choice(["gauss_outlier", "student_t"])), seed=int(r.integers(1, 1 << 30)))
+
+
+@pytest.mark.parametrize("case", range(N_CASES))
+def test_fused_random_shapes(orc, case, monkeypatch):
+    c = draw_case(case)
+    if c["cluster"]:
+        monkeypatch.setenv("VD_CLUSTER_SIZE", str(c["cluster"]))
+    d, N, B, cap = c["d"], c["N"], c["B"], c["cap"]
+    cache = new_cache(c["n_seq"], c["L"], c["H"], cap, d)
+    U, us, per_seq = cache.units, cache.unit_shape(), c["L"] * c["H"]
+    st = wl.TokenStream(c["gen"], U, d, device="cuda", seed=c["seed"])
+    wl.fill_rows(st, units_view(cache.k), units_view(cache.v), cap)
+    cache.len.copy_(torch.tensor(c["lens"], dtype=torch.int32))
+    rs = torch.zeros(us + (d,), dtype=torch.float64, device="cuda")
+    if c["mu"] == vd.VD_MU_RUNNING:
+        vd.vd_running_sum_init(cache, rs)
+    pos = pos_new = None
+    if c["holefill"]:
+        pos = torch.arange(cap, dtype=torch.int32, device="cuda").repeat(U).view(us + (cap,))
+        pos = pos.contiguous()
+    N_dev = (torch.tensor(c["budgets"], dtype=torch.int32, device="cuda")
+             if c["budgets"] else None)
+    Ns = c["budgets"] if c["budgets"] else [N] * c["n_seq"]
+    for event in range(2):
+        lens = cache.len.cpu().numpy().copy()
+        pre_k, pre_v = bits(units_view(cache.k)), bits(units_view(cache.v))
+        pre_pos = pos.view(U, cap).cpu().numpy().copy() if pos is not None else None
+        k_new, v_new = st.next(B)
+        k_new, v_new = k_new.view(us + (B, d)).contiguous(), v_new.view(us + (B, d)).contiguous()
+        kn, vn = bits(k_new.view(U, B, d)), bits(v_new.view(U, B, d))
+        if pos is not None:
+            pos_new = torch.full((c["n_seq"],), cap + 1000 * (event + 1), dtype=torch.int32,
+                                 device="cuda")
+        kept = torch.full(us + (N,), -7, dtype=torch.int32, device="cuda")
+        scores = torch.full(us + (cap,), float("nan"), device="cuda")
+        evicted = torch.full(us, -7, dtype=torch.int32, device="cuda")
+        rs_arg = rs if c["mu"] == vd.VD_MU_RUNNING else None
+        if c["two_call"]:
+            vd.vd_append(cache, k_new, v_new, B)
+            if c["decode"] and pos is not None:
+                vd.vd_evict_decode_holefill(cache, N, pos, pos_new, N_dev, c["var"], c["mu"],
+                                            rs_arg, evicted, kept, scores)
+            elif c["decode"]:
+                vd.vd_evict_decode(cache, N, N_dev, c["var"], c["mu"], rs_arg, evicted, kept,
+                                   scores)
+            elif pos is not None:
+                vd.vd_evict_block_holefill(cache, N, pos, pos_new, N_dev, B, c["var"], c["mu"],
+                                           rs_arg, kept, scores)
+            else:
+                vd.vd_evict_block(cache, N, N_dev, B, c["var"], c["mu"], rs_arg, kept, scores)
+        elif c["decode"]:
+            vd.vd_append_evict_decode(cache, k_new, v_new, N, N_dev, c["var"], c["mu"], rs_arg,
+                                      evicted, kept, scores, pos=pos, pos_first_new=pos_new)
+        else:
+            vd.vd_append_evict_block(cache, k_new, v_new, B, N, N_dev, c["var"], c["mu"], rs_arg,
+                                     kept, scores, pos=pos, pos_first_new=pos_new)
+        assert vd.vd_get_device_status() == 0, c
+        post_k, post_v = bits(units_view(cache.k)), bits(units_view(cache.v))
+        new_lens = cache.len.cpu().numpy()
+        kh, sh = kept.view(U, N).cpu().numpy(), scores.view(U, cap).cpu().numpy()
+        post_pos = pos.view(U, cap).cpu().numpy() if pos is not None else None
+        for u in range(U):
+            s = u // per_seq
+            len0 = int(lens[s])  # read before the call: the pre-append length
+            n, Nb = len0 + B, Ns[s]
+            assert new_lens[s] == min(n, Nb), (c, event, u)
+            # the rows the event saw: the cache's len0 rows, then the new ones
+            ek = np.concatenate([pre_k[u, :len0], kn[u]])
+            ev = np.concatenate([pre_v[u, :len0], vn[u]])
+            if pos is None:
+                check_event(orc, c["var"], ek, ev, post_k[u], post_v[u], n, Nb,
+                            kh[u] if n > Nb else None, sh[u] if n > Nb else None)
+            else:
+                ep = np.concatenate([pre_pos[u, :len0], int(pos_new[s]) + np.arange(B)])
+                check_holefill_event(orc, c["var"], ek, ev, ep.astype(np.int32), post_k[u],
+                                     post_v[u], post_pos[u], n, Nb, kh[u] if n > Nb else None,
+                                     sh[u] if n > Nb else None)
+        if c["mu"] == vd.VD_MU_RUNNING:
+            ref = torch.zeros_like(rs)
+            vd.vd_running_sum_init(cache, ref)
+            scale = units_view(cache.v).float().abs().sum(dim=1).max().item() + 1.0
+            assert torch.max(torch.abs(ref - rs)).item() <= 1e-12 * scale, (c, event)
