@@ -27,6 +27,7 @@ from vd_gpu import bits, check_event, new_cache, units_view
 pytestmark = pytest.mark.gpu
 HEAD_DIMS = [8, 16, 24, 40, 64, 72, 128, 136, 200, 256]
 N_CASES = 48
+N_MEDIUM = 8  # budgets of 1000-6000 tokens, the batched score paths' head dims
 
 
 @pytest.fixture(scope="module", autouse=True)
@@ -38,12 +39,12 @@ def _lib():
     assert vd.vd_get_device_status() == 0
 
 
-def draw_case(i):
-    r = np.random.default_rng(7919 * (i + 1))
-    d = int(r.choice(HEAD_DIMS))
+def draw_case(i, medium=False):
+    r = np.random.default_rng(7919 * (i + 1) + (104729 if medium else 0))
+    d = int(r.choice([64, 128, 256] if medium else HEAD_DIMS))
     decode = bool(r.random() < 0.35)
-    N = int(r.integers(1, 401))
-    B = 1 if decode else int(r.integers(1, 97))
+    N = int(r.integers(1000, 6001)) if medium else int(r.integers(1, 401))
+    B = 1 if decode else int(r.integers(1, 513 if medium else 97))
     n_seq, L, H = int(r.integers(1, 4)), int(r.integers(1, 3)), int(r.integers(1, 4))
     budgets = [int(r.integers(1, N + 1)) for _ in range(n_seq)] if r.random() < 0.3 else None
     lens = [int(r.integers(max(0, Nb - 3 * B), Nb + 1))
@@ -58,9 +59,12 @@ def draw_case(i):
                 gen=str(r.choice(["gauss_outlier", "student_t"])), seed=int(r.integers(1, 1 << 30)))
 
 
-@pytest.mark.parametrize("case", range(N_CASES))
+@pytest.mark.parametrize("case", [(i, False) for i in range(N_CASES)] +
+                         [(i, True) for i in range(N_MEDIUM)],
+                         ids=[f"small{i}" for i in range(N_CASES)] +
+                         [f"medium{i}" for i in range(N_MEDIUM)])
 def test_fused_random_shapes(orc, case, monkeypatch):
-    c = draw_case(case)
+    c = draw_case(*case)
     if c["cluster"]:
         monkeypatch.setenv("VD_CLUSTER_SIZE", str(c["cluster"]))
     d, N, B, cap = c["d"], c["N"], c["B"], c["cap"]
