@@ -15,7 +15,10 @@
 //             shuffle reduction of the squared deviation (L2), of the norm
 //             (Norm), or of the normalised difference (Dir, as
 //             1/2 |v/|v| - mean/|mean||^2, which equals 1 - cos without
-//             cancellation).  Scores become order-preserving uint32 keys.
+//             cancellation).  For d = 64, 128, 256 (L2, Norm) each lane keeps
+//             a batch of 8 rows' partial sums (packed f32x2 arithmetic) and
+//             the batch is reduced with a transposed butterfly
+//             (score_rows_fast).  Scores become order-preserving uint32 keys.
 //   3. select block prompt processing (N+B -> N): a 4-pass 8-bit radix select
 //             for the N-th largest key t; every CTA histograms only its own
 //             rows and the cluster adds the C histograms through DSMEM.
@@ -27,7 +30,8 @@
 //             perm[] (uint16): kept slots ascending in [0, N), then the
 //             evicted slots ascending.
 //   5. sum    running-sum mode: S += sum(appended rows) - sum(evicted rows)
-//             over the V columns this CTA moves, before it moves them.
+//             over the columns of the scored tensor (V, or K for the key-side
+//             rule) this CTA moves, before it moves them.
 //   6. move   K' = gather(K, perm), V' = gather(V, perm), in place, for the
 //             rows r = first evicted .. N-1 of this CTA's column slice.  Tiles
 //             of rows stream through the cp.async ring; tile t is stored only
@@ -36,6 +40,12 @@
 //             perm[r] >= r, a tile's destinations lie below every source a
 //             later tile reads, so the ascending order is hazard-free, and
 //             column slices make the CTAs of a unit independent.
+//
+// Template flags select the rest at compile time: DECODE (the arg-min path),
+// HF (hole-fill layout: ties broken by token position, and only the kept rows
+// at or above N move, into the evicted slots below N) and FUSED (the rows at
+// or above len are read from the caller's staging buffers and written only
+// if they survive: the append of Eq. block_processing fused into the event).
 //
 // Nothing waits on a flag; the only cross-CTA synchronisation is the hardware
 // cluster barrier, which every CTA of a cluster reaches the same number of
