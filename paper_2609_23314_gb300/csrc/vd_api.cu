@@ -230,15 +230,21 @@ bool cluster_allowed(int c, int d) {
 // smallest C with 0.85-1 waves or at least four, else the decode rule.
 // Hole-fill block eviction (moves few rows, so the select's cluster
 // synchronisation dominates and grows with C): the smallest C with at least
-// 0.85 of a wave.  With none such, the largest allowed C.  (Measured on
-// GB300: prefill_wide ordered C=8 (4.4 waves) 0.574 ms vs C=4 (2.2) 0.586;
-// hole-fill C=2 (1.1 waves) 0.205 vs C=4 0.216; decode C=1.)  Where no C
+// 0.85 of a wave.  With none such (few units), the largest allowed C that
+// leaves every CTA at least kMinRowsPerCta rows of the capacity, else the
+// smallest allowed C: below that, the cluster barriers cost more than the
+// split saves.  (Measured on GB300: prefill_wide ordered C=8 (4.4 waves)
+// 0.574 ms vs C=4 (2.2) 0.586; hole-fill C=2 (1.1 waves) 0.205 vs C=4
+// 0.216; decode C=1; two units of 160 rows C=1 16.8 us vs C=4 18.5, of 600
+// rows C=4 20.9 vs C=1 26.4, of 2400 rows C=8 27.9 vs C=1 75.7.)  Where no C
 // with 64-byte segments fits the shared memory (a large capacity at a small
 // head dim), the smallest C that fits.  want
 // (VD_CLUSTER_SIZE: 1, 2, 4, 8 or 16) overrides the choice, for tuning.
+constexpr int kMinRowsPerCta = 128;
+
 int choose_cluster(const void* kern, long long units, int d, int capacity, bool with_select,
                    bool holefill, int want, const DeviceState& st, size_t* smem_out) {
-  int chosen = 0, fallback = 0, largest = 0, narrow = 0;
+  int chosen = 0, fallback = 0, roomy = 0, smallest = 0, narrow = 0;
   for (int c = 1; c <= 16; c *= 2) {
     if (want >= 1 && c != want) continue;
     if ((d / 8 * 2) % c) continue;
@@ -256,7 +262,8 @@ int choose_cluster(const void* kern, long long units, int d, int capacity, bool 
       if (narrow == 0) narrow = c;
       continue;
     }
-    largest = c;
+    if (smallest == 0) smallest = c;
+    if ((capacity + c - 1) / c >= kMinRowsPerCta) roomy = c;
     const double waves = (double)(units * c) / ((double)st.sms * occ);
     const bool full_wave = waves >= 0.85 && waves <= 1.0;
     bool ok;
@@ -274,7 +281,8 @@ int choose_cluster(const void* kern, long long units, int d, int capacity, bool 
     }
     if (fallback == 0 && (full_wave || waves >= 2.0)) fallback = c;
   }
-  if (chosen == 0) chosen = fallback ? fallback : largest ? largest : narrow ? narrow : 1;
+  if (chosen == 0)
+    chosen = fallback ? fallback : roomy ? roomy : smallest ? smallest : narrow ? narrow : 1;
   *smem_out = vd::smem_layout(capacity, chosen, with_select).total;
   return chosen;
 }
