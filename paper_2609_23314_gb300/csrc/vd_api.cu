@@ -230,11 +230,12 @@ bool cluster_allowed(int c, int d) {
 // smallest C with 0.85-1 waves or at least four, else the decode rule.
 // Hole-fill block eviction (moves few rows, so the select's cluster
 // synchronisation dominates and grows with C): the smallest C with at least
-// 0.85 of a wave.  With none such (few units), the largest allowed C that
+// 0.7 of a wave (one short wave beats a long tail: prefill_wide C=1, 0.74
+// waves, 0.211-0.216 ms vs C=2, 1.47 waves, 0.216-0.221).  With none such (few units), the largest allowed C that
 // leaves every CTA at least kMinRowsPerCta rows of the capacity, else the
 // smallest allowed C: below that, the cluster barriers cost more than the
 // split saves.  (Measured on GB300: prefill_wide ordered C=8 (4.4 waves)
-// 0.574 ms vs C=4 (2.2) 0.586; hole-fill C=2 (1.1 waves) 0.205 vs C=4
+// 0.574 ms vs C=4 (2.2) 0.586; hole-fill C=2 (1.47 waves) 0.205 vs C=4
 // 0.216; decode C=1; two units of 160 rows C=1 16.8 us vs C=4 18.5, of 600
 // rows C=4 20.9 vs C=1 26.4, of 2400 rows C=8 27.9 vs C=1 75.7.)  Where no C
 // with 64-byte segments fits the shared memory (a large capacity at a small
@@ -270,7 +271,7 @@ int choose_cluster(const void* kern, long long units, int d, int capacity, bool 
     if (want >= 1)
       ok = true;
     else if (with_select && holefill)
-      ok = waves >= 0.85;
+      ok = waves >= 0.7;
     else if (with_select)
       ok = full_wave || waves >= 4.0;
     else
