@@ -230,8 +230,10 @@ bool cluster_allowed(int c, int d) {
 // smallest C with 0.85-1 waves or at least four, else the decode rule.
 // Hole-fill block eviction (moves few rows, so the select's cluster
 // synchronisation dominates and grows with C): the smallest C with at least
-// 0.7 of a wave (one short wave beats a long tail: prefill_wide C=1, 0.74
-// waves, 0.211-0.216 ms vs C=2, 1.47 waves, 0.216-0.221).  With none such (few units), the largest allowed C that
+// 0.4 of a wave (one short wave beats a long tail and more cluster barriers:
+// prefill_wide C=1, 0.74 waves, 0.211-0.216 ms vs C=2, 1.47 waves,
+// 0.216-0.221; prefill_gqa8b C=1, 0.47 waves, 0.064 ms vs C=2, 0.95 waves,
+// 0.069).  With none such (few units), the largest allowed C that
 // leaves every CTA at least kMinRowsPerCta rows of the capacity, else the
 // smallest allowed C: below that, the cluster barriers cost more than the
 // split saves.  (Measured on GB300: prefill_wide ordered C=8 (4.4 waves)
@@ -271,7 +273,7 @@ int choose_cluster(const void* kern, long long units, int d, int capacity, bool 
     if (want >= 1)
       ok = true;
     else if (with_select && holefill)
-      ok = waves >= 0.7;
+      ok = waves >= 0.4;
     else if (with_select)
       ok = full_wave || waves >= 4.0;
     else
