@@ -142,3 +142,94 @@ def test_fused_random_shapes(orc, case, monkeypatch):
             vd.vd_running_sum_init(cache, ref)
             scale = units_view(cache.v).float().abs().sum(dim=1).max().item() + 1.0
             assert torch.max(torch.abs(ref - rs)).item() <= 1e-12 * scale, (c, event)
+
+
+N_EX = 24  # vd_evict_block_ex: key-side rule, attention weights, sigma by-product
+
+
+def draw_ex(i):
+    r = np.random.default_rng(31337 * (i + 1))
+    d = int(r.choice(HEAD_DIMS))
+    N, B = int(r.integers(1, 401)), int(r.integers(1, 97))
+    n_seq, L, H = int(r.integers(1, 4)), int(r.integers(1, 3)), int(r.integers(1, 4))
+    var = int(r.integers(0, 3))
+    allowed = [c for c in (1, 2, 4, 8, 16) if (2 * (d // 8)) % c == 0]
+    return dict(d=d, N=N, B=B, n_seq=n_seq, L=L, H=H,
+                lens=[int(r.integers(max(0, N - 2 * B), N + 1)) for _ in range(n_seq)],
+                cap=N + B + int(r.integers(0, 17)), var=var, keys=bool(r.random() < 0.5),
+                weighted=bool(r.random() < 0.4), disp=var == 0 and bool(r.random() < 0.5),
+                mu=int(r.integers(0, 2)),
+                cluster=int(r.choice(allowed)) if r.random() < 0.5 else 0,
+                gen=str(r.choice(["gauss_outlier", "student_t"])), seed=int(r.integers(1, 1 << 30)))
+
+
+@pytest.mark.parametrize("case", range(N_EX))
+def test_ex_random_options(orc, case, monkeypatch):
+    """One block event through vd_evict_block_ex with random scoring options:
+    scores of the scored tensor (K for the key-side rule) within the parity
+    tolerance (weighted: scaled by the factor a/(1 - a), App. A), the kept
+    set outside near ties, bit-exact gathers, sigma of the plain L2 scores
+    for the units that evicted, and the running sum of the scored tensor."""
+    import test_gpu_extensions as tx
+    from vd_gpu import score_tolerance
+    tx._ORC = orc
+    c = draw_ex(case)
+    if c["cluster"]:
+        monkeypatch.setenv("VD_CLUSTER_SIZE", str(c["cluster"]))
+    d, N, B, cap, var = c["d"], c["N"], c["B"], c["cap"], c["var"]
+    cache = new_cache(c["n_seq"], c["L"], c["H"], cap, d)
+    U, us, per_seq = cache.units, cache.unit_shape(), c["L"] * c["H"]
+    st = wl.TokenStream(c["gen"], U, d, device="cuda", seed=c["seed"])
+    wl.fill_rows(st, units_view(cache.k), units_view(cache.v), cap)
+    cache.len.copy_(torch.tensor(c["lens"], dtype=torch.int32))
+    rs = torch.zeros(us + (d,), dtype=torch.float64, device="cuda")
+    running = c["mu"] == vd.VD_MU_RUNNING
+    if running:
+        vd.vd_running_sum_init_ex(cache, c["keys"], rs)
+    k_new, v_new = st.next(B)
+    vd.vd_append(cache, k_new.view(us + (B, d)).contiguous(), v_new.view(us + (B, d)).contiguous(), B)
+    lens = cache.len.cpu().numpy().copy()
+    pre_k, pre_v = bits(units_view(cache.k)), bits(units_view(cache.v))
+    attn = None
+    if c["weighted"]:
+        g = torch.Generator(device="cuda").manual_seed(c["seed"] % 100003)
+        attn = torch.rand(us + (cap,), generator=g, device="cuda") * 0.9
+        attn[..., ::17] = 0.0
+    kept = torch.full(us + (N,), -7, dtype=torch.int32, device="cuda")
+    scores = torch.full(us + (cap,), float("nan"), device="cuda")
+    sigma = torch.full(us, -1.0, device="cuda") if c["disp"] else None
+    vd.vd_evict_block_ex(cache, N, None, B, var, c["mu"], rs if running else None, c["keys"],
+                         attn, kept, scores, sigma)
+    assert vd.vd_get_device_status() == 0, c
+    post_k, post_v = bits(units_view(cache.k)), bits(units_view(cache.v))
+    kh, sh = kept.view(U, N).cpu().numpy(), scores.view(U, cap).cpu().numpy()
+    a_h = attn.view(U, cap).cpu().numpy().astype(np.float64) if attn is not None else None
+    sg = sigma.view(U).cpu().numpy() if sigma is not None else None
+    for u in range(U):
+        n = int(lens[u // per_seq])
+        src = pre_k[u, :n] if c["keys"] else pre_v[u, :n]
+        if n <= N:
+            assert np.array_equal(post_k[u, :n], pre_k[u, :n])
+            assert np.array_equal(post_v[u, :n], pre_v[u, :n])
+            if sg is not None:
+                assert sg[u] == -1.0, (c, u)
+            continue
+        if a_h is None:
+            s_ora = orc.scores(src, var)
+            tol = score_tolerance(var, s_ora, src, orc.mean(src))
+        else:
+            s_ora = orc.scores_weighted(src, a_h[u, :n], var)
+            f = a_h[u, :n] / (1.0 - a_h[u, :n])
+            tol = (score_tolerance(var, orc.scores(src, var), src, orc.mean(src)) * f
+                   + 2e-7 * np.abs(s_ora))
+        tx.check_scored_event(s_ora, tol, pre_k[u], pre_v[u], post_k[u], post_v[u], n, N, kh[u],
+                              sh[u])
+        if sg is not None:
+            want = orc.dispersion(src)
+            assert abs(sg[u] - want) <= 1e-5 * want + 1e-6, (c, u, sg[u], want)
+    if running:
+        ref = torch.zeros_like(rs)
+        vd.vd_running_sum_init_ex(cache, c["keys"], ref)
+        t = units_view(cache.k if c["keys"] else cache.v)
+        scale = t.float().abs().sum(dim=1).max().item() + 1.0
+        assert torch.max(torch.abs(ref - rs)).item() <= 1e-12 * scale, c
