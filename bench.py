@@ -636,6 +636,24 @@ def run_e2e(w, steps, device):
     return start.elapsed_time(stop)
 
 
+def h2d_rate(w, nbytes, reps=5):
+    """GB/s of one step's host-to-device copies alone (the e2e buffers, no
+    eviction running): the link rate the e2e number is measured against."""
+    import torch
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    times = []
+    for i in range(reps + 1):
+        torch.cuda.synchronize()
+        a.record()
+        w.e2e_h2d(i, 0)
+        b.record()
+        torch.cuda.synchronize()
+        if i:
+            times.append(a.elapsed_time(b))
+    times.sort()
+    return nbytes / (times[len(times) // 2] / 1e3) / 1e9
+
+
 def measure_gpu(w, steps, warmup, device, e2e_steps):
     import torch
     for _ in range(warmup):
@@ -664,13 +682,14 @@ def measure_gpu(w, steps, warmup, device, e2e_steps):
     moved = w.moved_rows(kept)
     # end to end through the C ABI with host buffers
     bi, bo = w.e2e_setup(e2e_steps)
+    link_gbs = h2d_rate(w, bi)
     run_e2e(w, min(3, warmup), device)
     e2e_ms = run_e2e(w, e2e_steps, device)
     status = w.vd.vd_get_device_status()
     if status != 0:
         raise RuntimeError(f"device status {status}: {w.vd.vd_status_string(status)}")
     return dict(step_ms=step_ms, kern_ms=kern_ms, moved=moved, clocks=clk, e2e_ms=e2e_ms,
-                bi=bi, bo=bo)
+                bi=bi, bo=bo, link_gbs=link_gbs)
 
 
 def graph_step_us(w, steps, device):
@@ -849,7 +868,8 @@ def run_vd(args):
             "workload": name, "w": w, "m": m, "step_ms": step_ms, "kern_ms": kern_ms,
             "value": tok * ws / (step_ms / 1e3),
             "e2e": {"value": tok * ws / (e2e_ms / 1e3), "unit": UNIT,
-                    "h2d_bytes_per_step": m["bi"], "d2h_bytes_per_step": m["bo"]},
+                    "h2d_bytes_per_step": m["bi"], "d2h_bytes_per_step": m["bo"],
+                    "h2d_gbs_alone": m["link_gbs"]},
             "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                          "frac": achieved / peak,
                          "traffic": ncu_traffic(name, layout, separate=not getattr(w, "fused", True))
