@@ -13,8 +13,9 @@ and larger than L2.  Prints one JSON line (rank 0):
   roofline    the fused eviction kernel: algorithmic bytes per launch / its
               CUDA-event duration, against the measured HBM copy bandwidth
   e2e         the same metric through the C ABI with the step's new K/V rows
-              copied from pinned host memory and the step's result (kept or
-              evicted slots) copied back, every step
+              copied from pinned host memory (a pool of E2E_POOL staging
+              buffers) and the step's result (kept or evicted slots) copied
+              back, every step
   cpu_baseline  the fp64 CPU oracle on a bounded sample of the same events
   secondary   the largest decode workload measured the same way (default run)
 
@@ -43,6 +44,11 @@ METRIC = "cache tokens scored+compacted/s; HBM GB/s as % of GB300 peak per evict
 UNIT = "head-tokens/s"
 FALLBACK_HBM_GBS = 6800.0
 L2_BYTES = 129 * 2 ** 20
+# pinned host staging buffers the e2e run cycles through, as a caller's
+# staging pool would: copies from 50 distinct 88 MB pinned blocks (4.4 GB)
+# ran 4-6x slower than from 8 on the same GB300, although each copy alone
+# runs at ~204 GB/s
+E2E_POOL = 8
 
 
 # ---------------------------------------------------------------------------
@@ -681,7 +687,7 @@ def measure_gpu(w, steps, warmup, device, e2e_steps):
     kern_ms = sum(a.elapsed_time(b) for a, b in evs) / steps
     moved = w.moved_rows(kept)
     # end to end through the C ABI with host buffers
-    bi, bo = w.e2e_setup(e2e_steps)
+    bi, bo = w.e2e_setup(min(e2e_steps, E2E_POOL))
     link_gbs = h2d_rate(w, bi)
     run_e2e(w, min(3, warmup), device)
     e2e_ms = run_e2e(w, e2e_steps, device)
