@@ -597,11 +597,15 @@ __device__ __forceinline__ void cluster_build_perm(const uint32_t* keys, int r0,
 // source row perm[r] (or r + 1 when perm is null: the decode shift).  A
 // source at or above n (impossible for a consistent slot list) is not read
 // and is recorded as kStInternal (its row then holds unspecified bytes).
-template <class Ring>
+// STAGED (fused append): sources at or above first_stage are rows of the
+// staging buffers kn / vn ([B][d] per unit) and stream through the same
+// ring; they are never cache rows, so the order stays hazard-free.
+template <class Ring, bool STAGED>
 __device__ __forceinline__ void compact_slice(uint16_t* kb, uint16_t* vb, int d, int chunk0,
                                               int cps, int r_begin, int r_end, int n,
                                               const uint16_t* perm, unsigned* status,
-                                              uint32_t ring) {
+                                              uint32_t ring, const uint16_t* kn,
+                                              const uint16_t* vn, int first_stage) {
   const int tid = threadIdx.x;
   const int d8 = d >> 3;
   const int rs = kThreads / cps;
@@ -609,6 +613,8 @@ __device__ __forceinline__ void compact_slice(uint16_t* kb, uint16_t* vb, int d,
   const int my_ch = chunk0 + tid % cps;
   const int my_off = tid / cps;
   uint16_t* col = my_ch < d8 ? kb + my_ch * 8 : vb + (my_ch - d8) * 8;
+  const uint16_t* scol = nullptr;  // this thread's column of the staging rows
+  if constexpr (STAGED) scol = my_ch < d8 ? kn + my_ch * 8 : vn + (my_ch - d8) * 8;
   constexpr int kRingStages = Ring::kStages, kRingItems = Ring::kItems;
   const int tile = rs * kRingItems;
   const int ntiles = r_end > r_begin ? (r_end - r_begin + tile - 1) / tile : 0;
@@ -623,10 +629,14 @@ __device__ __forceinline__ void compact_slice(uint16_t* kb, uint16_t* vb, int d,
         const int r = r_begin + t * tile + u * rs + my_off;
         if (on && r < r_end) {
           const int src = perm ? (int)perm[r] : r + 1;
-          if (src < n)
-            cp_async16(slot(t % kRingStages, u), col + (size_t)src * d);
-          else
+          if (src < n) {
+            const uint16_t* sp = col + (size_t)src * d;
+            if constexpr (STAGED)
+              if (src >= first_stage) sp = scol + (size_t)(src - first_stage) * d;
+            cp_async16(slot(t % kRingStages, u), sp);
+          } else {
             record_status(status, kStInternal);
+          }
         }
       }
     }
@@ -666,42 +676,6 @@ __device__ __forceinline__ void copy_new_rows(uint16_t* kb, uint16_t* vb, const 
         const int i = it / cps, c = chunk0 + it % cps;
         q[k] = ld_cg16((c < d8 ? kn + c * 8 : vn + (c - d8) * 8) + (size_t)i * d);
         dstp[k] = (c < d8 ? kb + c * 8 : vb + (c - d8) * 8) + (size_t)(first + i) * d;
-      }
-    }
-#pragma unroll
-    for (int k = 0; k < U; ++k)
-      if (dstp[k]) st16(dstp[k], q[k]);
-  }
-}
-
-// Fused append, ordered layout: cache rows [r_lo, r_hi) of this CTA's column
-// slice take staging row stage_of(r) (kept new rows; their slots follow
-// every slot fed from the cache, because kept slots are ascending).  A
-// staging index outside [0, B) (never expected) is skipped and recorded.
-template <class StageOf>
-__device__ __forceinline__ void copy_staged_rows(uint16_t* kb, uint16_t* vb, const uint16_t* kn,
-                                                 const uint16_t* vn, int d, int chunk0, int cps,
-                                                 int r_lo, int r_hi, int B, StageOf stage_of,
-                                                 unsigned* status) {
-  const int d8 = d >> 3;
-  const int items = (r_hi - r_lo) * cps;
-  constexpr int U = 4;  // loads in flight per thread before the stores
-  for (int base = threadIdx.x; base < items; base += kThreads * U) {
-    uint4 q[U];
-    uint16_t* dstp[U];
-#pragma unroll
-    for (int k = 0; k < U; ++k) {
-      const int it = base + k * kThreads;
-      dstp[k] = nullptr;
-      if (it < items) {
-        const int r = r_lo + it / cps, c = chunk0 + it % cps;
-        const int i = stage_of(r);
-        if ((unsigned)i < (unsigned)B) {
-          q[k] = ld_cg16((c < d8 ? kn + c * 8 : vn + (c - d8) * 8) + (size_t)i * d);
-          dstp[k] = (c < d8 ? kb + c * 8 : vb + (c - d8) * 8) + (size_t)r * d;
-        } else {
-          record_status(status, kStInternal);
-        }
       }
     }
 #pragma unroll
@@ -1184,33 +1158,12 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
 
   // ---- 6. in-place compaction of this CTA's column slice ---------------
   if constexpr (!HF) {
-    // fused append: kept new rows below the budget are written too.  Their
-    // sources are the staging rows, and they occupy the suffix [r_star, Nb)
-    // of the compaction range (kept slots ascend); the cache-fed part runs
-    // first, then (after a barrier: it may still read rows of that suffix)
-    // the staged rows are copied in.
-    auto src_of = [&](int r) { return DECODE ? r + 1 : (int)perm[r]; };
+    // fused append: kept new rows below the budget are written too, read
+    // from the staging rows in the same stream (their slots, the suffix of
+    // the kept list, come last)
     const int r_begin = min(e_first, first_stage);
-    int r_star = Nb;
-    if (fused) {
-      if (tid == 0) {
-        int lo = r_begin, hi = Nb;
-        while (lo < hi) {
-          const int mid = (lo + hi) >> 1;
-          if (src_of(mid) < first_stage) lo = mid + 1; else hi = mid;
-        }
-        S.holes = lo;
-      }
-      __syncthreads();
-      r_star = S.holes;
-    }
-    compact_slice<Ring>(kb, vb, d, chunk0, cps, r_begin, r_star, n, DECODE ? nullptr : perm,
-                        a.status, ring);
-    if (fused && r_star < Nb) {
-      __syncthreads();
-      copy_staged_rows(kb, vb, knu, vnu, d, chunk0, cps, r_star, Nb, a.B,
-                       [&](int r) { return src_of(r) - first_stage; }, a.status);
-    }
+    compact_slice<Ring, FUSED>(kb, vb, d, chunk0, cps, r_begin, Nb, n, DECODE ? nullptr : perm,
+                               a.status, ring, knu, vnu, first_stage);
   } else {
     // hole-fill: the kept rows at or above N move into the evicted slots
     // below N, in ascending order (movers: the tail of the kept list; holes:
