@@ -1,9 +1,9 @@
 """Properties of the CUDA path that the mathematics fixes, checked on the GPU
 without the oracle: positive homogeneity of the scores (Sec. 3.2: L2 and Norm
 scale with the values, Dir does not), permutation equivariance of the kept
-set (Eq. eviction ranks tokens, not slots), and translation invariance of
-the L2 score (a constant shift of every value moves the mean with it).
-Needs a GB300."""
+set (Eq. eviction ranks tokens, not slots), translation invariance of the
+L2 score (a constant shift of every value moves the mean with it), and the
+L2 score as the uniform-attention disturbance of Sec. 3.3.  Needs a GB300."""
 from __future__ import annotations
 
 import numpy as np
@@ -123,3 +123,27 @@ def test_translation_invariance_of_l2():
     assert np.array_equal(k1, k2)
     # the same tokens' K rows were kept, in the same order
     assert torch.equal(cache.k, shifted.k)
+
+
+def test_scores_equal_the_uniform_attention_disturbance():
+    """Sec. 3.3: under uniform attention the output is the mean of the cached
+    values, and removing token j moves it by (mean - v_j) / (n - 1).  Brute
+    force in fp64 (recompute the mean without each token) gives
+    (n - 1) * |o - o_without_j| = s_j: the GPU's L2 scores match it within the
+    parity tolerance and rank the tokens the same way outside near ties."""
+    n, d, units, N = 96, 64, 2, 64
+    cache = filled(n, d, seed=19, units=units)
+    s_gpu = scores_of(cache, vd.VD_SCORE_L2)[:, :n].double().cpu().numpy()
+    vals = units_view(cache.v)[:, :n].double().cpu().numpy()
+    for u in range(units):
+        v = vals[u]
+        o = v.mean(axis=0)
+        disturb = np.array([(n - 1) * np.linalg.norm(o - np.delete(v, j, axis=0).mean(axis=0))
+                            for j in range(n)])
+        tol = 1e-5 * disturb + 2e-6 * (np.linalg.norm(v, axis=1) + np.linalg.norm(o))
+        assert np.all(np.abs(s_gpu[u] - disturb) <= tol)
+        top_gpu = np.sort(np.argsort(-s_gpu[u], kind="stable")[:N])
+        top_bf = np.sort(np.argsort(-disturb, kind="stable")[:N])
+        diff = np.setxor1d(top_gpu, top_bf)
+        if diff.size:
+            assert np.all(near_tie_band(disturb, N)[diff])
