@@ -232,6 +232,22 @@ vd_status vd_evict_block_ex(const vd_cache* c, int32_t N, const int32_t* N_dev, 
                             int32_t score_keys, const float* attn, int32_t* kept_idx_out,
                             float* scores_out, float* dispersion_out, vd_stream_t stream);
 
+/* vd_append followed by vd_evict_block_ex in one launch, as
+ * vd_append_evict_block is for vd_evict_block (one step of Sec. 2.2,
+ * Eq. block_processing, with the scoring options above): k_new, v_new are
+ * bf16 device [n_seq][n_layer][n_kv_head][B][head_dim], 16-byte aligned,
+ * read straight from the caller's buffers, and only surviving rows are
+ * written.  len does not count the new rows before the call; during the
+ * event they occupy slots len .. len + B - 1, which is where attn, the
+ * scores and the kept slots refer to them.  Results are identical to
+ * vd_append followed by vd_evict_block_ex.  Ordered layout; errors as
+ * vd_append_evict_block and vd_evict_block_ex. */
+vd_status vd_append_evict_block_ex(const vd_cache* c, const void* k_new, const void* v_new,
+                                   int32_t B, int32_t N, const int32_t* N_dev, vd_variant var,
+                                   vd_mu_mode mu, double* running_sum, int32_t score_keys,
+                                   const float* attn, int32_t* kept_idx_out, float* scores_out,
+                                   float* dispersion_out, vd_stream_t stream);
+
 /* Hole-fill layout (not in the paper; its eviction rule with a cache layout
  * that moves as few rows as possible).  Same policy as vd_evict_block /
  * vd_evict_decode (Sec. 2.1, Eq. eviction; Sec. 2.2, Eq. block_processing),

@@ -21,7 +21,7 @@ import threading
 __all__ = [
     "VD_SCORE_L2", "VD_SCORE_DIR", "VD_SCORE_NORM", "VD_MU_RECOMPUTE", "VD_MU_RUNNING",
     "VdError", "Cache", "vd_score", "vd_score_ex", "vd_evict_block", "vd_evict_block_ex",
-    "vd_append_evict_block", "vd_append_evict_decode",
+    "vd_append_evict_block", "vd_append_evict_block_ex", "vd_append_evict_decode",
     "vd_evict_decode",
     "vd_evict_block_holefill", "vd_evict_decode_holefill", "vd_append",
     "vd_running_sum_init", "vd_running_sum_init_ex", "vd_workspace_size", "vd_status_string",
@@ -76,6 +76,8 @@ def load_library() -> ctypes.CDLL:
             lib.vd_evict_decode_holefill.argtypes = [cp, I32, P, S, S, P, P, P, P, P, P, P]
             lib.vd_score_ex.argtypes = [cp, S, S, P, I32, P, P, P]
             lib.vd_evict_block_ex.argtypes = [cp, I32, P, I32, S, S, P, I32, P, P, P, P, P]
+            lib.vd_append_evict_block_ex.argtypes = [cp, P, P, I32, I32, P, S, S, P, I32, P, P, P,
+                                                     P, P]
             lib.vd_append.argtypes = [cp, P, P, I32, P]
             lib.vd_running_sum_init.argtypes = [cp, P, P]
             lib.vd_running_sum_init_ex.argtypes = [cp, I32, P, P]
@@ -85,7 +87,7 @@ def load_library() -> ctypes.CDLL:
             lib.vd_status_string.restype = ctypes.c_char_p
             lib.vd_get_device_status.argtypes = [P]
             for f in ("vd_score", "vd_score_ex", "vd_evict_block_ex", "vd_evict_block",
-                      "vd_append_evict_block", "vd_append_evict_decode",
+                      "vd_append_evict_block", "vd_append_evict_block_ex", "vd_append_evict_decode",
                       "vd_evict_decode", "vd_evict_block_holefill",
                       "vd_evict_decode_holefill", "vd_append", "vd_running_sum_init",
                       "vd_running_sum_init_ex",
@@ -305,6 +307,33 @@ def vd_evict_block_ex(cache: Cache, N: int, N_dev=None, B: int = 0, variant: int
                                             int(mu), args[1], int(bool(score_keys)), args[2],
                                             args[3], args[4], args[5], _stream(stream)),
            "vd_evict_block_ex")
+
+
+def vd_append_evict_block_ex(cache: Cache, k_new, v_new, B: int, N: int, N_dev=None,
+                             variant: int = VD_SCORE_L2, mu: int = VD_MU_RECOMPUTE,
+                             running_sum=None, score_keys: bool = False, attn=None,
+                             kept_idx_out=None, scores_out=None, dispersion_out=None,
+                             stream=None) -> None:
+    """vd_append followed by vd_evict_block_ex in one launch; k_new, v_new:
+    bf16 [n_seq, n_layer, n_kv_head, B, head_dim], read straight from the
+    caller's buffers (attn covers the new rows at slots len .. len + B - 1)."""
+    torch = _torch()
+    us = cache.unit_shape()
+    shape = us + (int(B), cache.head_dim)
+    args = (
+        _ptr(k_new, torch.bfloat16, shape, "k_new", cache.device),
+        _ptr(v_new, torch.bfloat16, shape, "v_new", cache.device),
+        _ptr(N_dev, torch.int32, (cache.n_seq,), "N_dev", cache.device),
+        _ptr(running_sum, torch.float64, us + (cache.head_dim,), "running_sum", cache.device),
+        _ptr(attn, torch.float32, us + (cache.capacity,), "attn", cache.device),
+        _ptr(kept_idx_out, torch.int32, us + (int(N),), "kept_idx_out", cache.device),
+        _ptr(scores_out, torch.float32, us + (cache.capacity,), "scores_out", cache.device),
+        _ptr(dispersion_out, torch.float32, us, "dispersion_out", cache.device),
+    )
+    _check(load_library().vd_append_evict_block_ex(
+        cache.ref(), args[0], args[1], int(B), int(N), args[2], int(variant), int(mu), args[3],
+        int(bool(score_keys)), args[4], args[5], args[6], args[7], _stream(stream)),
+        "vd_append_evict_block_ex")
 
 
 def vd_evict_block_holefill(cache: Cache, N: int, pos, pos_first_new, N_dev=None, B: int = 0,

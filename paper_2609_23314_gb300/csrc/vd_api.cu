@@ -482,6 +482,16 @@ vd_status vd_evict_block_ex(const vd_cache* c, int32_t N, const int32_t* N_dev, 
              attn, dispersion_out);
 }
 
+vd_status vd_append_evict_block_ex(const vd_cache* c, const void* k_new, const void* v_new,
+                                   int32_t B, int32_t N, const int32_t* N_dev, vd_variant var,
+                                   vd_mu_mode mu, double* running_sum, int32_t score_keys,
+                                   const float* attn, int32_t* kept_idx_out, float* scores_out,
+                                   float* dispersion_out, vd_stream_t stream) {
+  return run(c, N, N_dev, B, var, mu, running_sum, nullptr, kept_idx_out, scores_out,
+             reinterpret_cast<cudaStream_t>(stream), false, false, nullptr, nullptr, score_keys,
+             attn, dispersion_out, k_new, v_new);
+}
+
 vd_status vd_evict_block_holefill(const vd_cache* c, int32_t N, const int32_t* N_dev, int32_t B,
                                   vd_variant var, vd_mu_mode mu, double* running_sum,
                                   int32_t* pos, const int32_t* pos_first_new,

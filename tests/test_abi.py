@@ -110,6 +110,15 @@ def test_scoring_options_rejected_before_launch(lib):
                                      None, None, None) == 2
     assert lib.vd_append_evict_block(ref, 0x100, 0x200, 4, 16, None, 0, 0, None, 0x300, None,
                                      None, None, None) == 1            # one position array
+    # the fused form of the scoring options: the same checks as both halves
+    assert lib.vd_append_evict_block_ex(ref, 0x100, None, 4, 16, None, 0, 0, None, 0, None,
+                                        None, None, None, None) == 1
+    assert lib.vd_append_evict_block_ex(ref, 0x108, 0x200, 4, 16, None, 0, 0, None, 0, None,
+                                        None, None, None, None) == 2
+    assert lib.vd_append_evict_block_ex(ref, 0x100, 0x200, 4, 16, None, 1, 0, None, 0, None,
+                                        None, None, 0x40, None) == 1   # sigma needs L2
+    assert lib.vd_append_evict_block_ex(ref, 0x100, 0x200, 4, 16, None, 0, 1, None, 1, None,
+                                        None, None, None, None) == 1   # running, no sum
     # the hole-fill layout needs both position arrays
     assert lib.vd_evict_block_holefill(ref, 16, None, 4, 0, 0, None, 0x40, None, None, None,
                                        None) == 1

@@ -350,3 +350,42 @@ def test_fused_per_sequence_budgets():
         n = ca.len.cpu().tolist()[u // per_seq]
         assert torch.equal(units_view(ca.k)[u, :n].view(torch.int16), units_view(cb.k)[u, :n].view(torch.int16))
         assert torch.equal(units_view(ca.v)[u, :n].view(torch.int16), units_view(cb.v)[u, :n].view(torch.int16))
+
+
+@pytest.mark.parametrize("var", VARS, ids=VAR_IDS)
+@pytest.mark.parametrize("keys", [False, True], ids=["values", "keys"])
+@pytest.mark.parametrize("weighted", [False, True], ids=["plain", "weighted"])
+@pytest.mark.parametrize("mu", [vd.VD_MU_RECOMPUTE, vd.VD_MU_RUNNING], ids=["recompute", "running"])
+def test_fused_scoring_options_match_two_calls(var, keys, weighted, mu):
+    """vd_append_evict_block_ex against vd_append + vd_evict_block_ex: the
+    key-side rule, attention weights over the new rows' slots, sigma (L2) and
+    either mean give bit-identical kept slots, scores, rows, lengths, running
+    sums and sigma."""
+    d, N, B = 128, 300, 64
+    cache, k_new, v_new = setup(d, N, B, [N, N - 40, 100], seed=311 + 7 * var)
+    us = cache.unit_shape()
+    attn = None
+    if weighted:
+        g = torch.Generator(device="cuda").manual_seed(3)
+        attn = torch.rand(us + (cache.capacity,), generator=g, device="cuda") * 0.9
+    out = []
+    for fused in (False, True):
+        c = vd.Cache(cache.k.clone(), cache.v.clone(), cache.len.clone())
+        rs = None
+        if mu == vd.VD_MU_RUNNING:
+            rs = torch.zeros(us + (d,), dtype=torch.float64, device="cuda")
+            vd.vd_running_sum_init_ex(c, keys, rs)
+        kept = torch.full(us + (N,), -7, dtype=torch.int32, device="cuda")
+        scores = torch.full(us + (cache.capacity,), float("nan"), device="cuda")
+        sigma = torch.full(us, -1.0, device="cuda") if var == oracle.L2 else None
+        if fused:
+            vd.vd_append_evict_block_ex(c, k_new, v_new, B, N, None, var, mu, rs, keys, attn,
+                                        kept, scores, sigma)
+        else:
+            vd.vd_append(c, k_new, v_new, B)
+            vd.vd_evict_block_ex(c, N, None, B, var, mu, rs, keys, attn, kept, scores, sigma)
+        assert vd.vd_get_device_status() == 0
+        out.append(((c, rs, kept, scores), sigma))
+    assert_same(out[0][0], out[1][0])
+    if out[0][1] is not None:
+        assert torch.equal(out[0][1], out[1][1])
