@@ -242,8 +242,9 @@ class Prefill:
         every timed event appends rows the cache has not seen.  layout
         "holefill" uses vd_evict_block_holefill with a token-position array.
         The step is one vd_append_evict_block call (the new block read
-        straight from its buffer) in either layout; separate_append and the
-        scoring options append with vd_append first."""
+        straight from its buffer) in either layout, and one
+        vd_append_evict_block_ex call with the scoring options;
+        separate_append appends with vd_append first."""
         import torch
         import paper_2609_23314_gb300 as vd
         from paper_2609_23314_gb300 import workloads as wl
@@ -287,7 +288,7 @@ class Prefill:
             self.attn = torch.rand(us + (self.cap,), generator=g, device=device) * 0.9
         # per-unit sigma (Sec. 3.1) of the pre-eviction rows, from the score pass
         self.sigma = torch.empty(us, device=device) if dispersion else None
-        self.fused = not (separate_append or score_keys or weighted or dispersion)
+        self.fused = not separate_append
         if self.fused:
             self.launches_per_step = 2     # fused append + evict, len update
         self.pending = None                # the block the next fused call appends
@@ -309,7 +310,14 @@ class Prefill:
             self.vd.vd_append(self.cache, k, v, self.B)
 
     def evict(self, kept=None, scores=None):
-        if self.fused:
+        options = self.score_keys or self.attn is not None or self.sigma is not None
+        if self.fused and options:
+            k, v = self.pending
+            self.vd.vd_append_evict_block_ex(self.cache, k, v, self.B, self.N, None, self.variant,
+                                             self.mu, self.rs if self.mu else None,
+                                             self.score_keys, self.attn, kept, scores,
+                                             self.sigma)
+        elif self.fused:
             k, v = self.pending
             hf = {}
             if self.holefill:
@@ -323,7 +331,7 @@ class Prefill:
             self.vd.vd_evict_block_holefill(self.cache, self.N, self.pos, pn, None, self.B,
                                             self.variant, self.mu, self.rs if self.mu else None,
                                             kept, scores)
-        elif self.score_keys or self.attn is not None or self.sigma is not None:
+        elif options:
             self.vd.vd_evict_block_ex(self.cache, self.N, None, self.B, self.variant, self.mu,
                                       self.rs if self.mu else None, self.score_keys, self.attn,
                                       kept, scores, self.sigma)
