@@ -160,12 +160,14 @@ def draw_ex(i):
                 weighted=bool(r.random() < 0.4), disp=var == 0 and bool(r.random() < 0.5),
                 mu=int(r.integers(0, 2)),
                 cluster=int(r.choice(allowed)) if r.random() < 0.5 else 0,
-                gen=str(r.choice(["gauss_outlier", "student_t"])), seed=int(r.integers(1, 1 << 30)))
+                gen=str(r.choice(["gauss_outlier", "student_t"])), seed=int(r.integers(1, 1 << 30)),
+                fused=bool(r.random() < 0.5))
 
 
 @pytest.mark.parametrize("case", range(N_EX))
 def test_ex_random_options(orc, case, monkeypatch):
-    """One block event through vd_evict_block_ex with random scoring options:
+    """One block event through vd_evict_block_ex (after vd_append) or
+    vd_append_evict_block_ex with random scoring options:
     scores of the scored tensor (K for the key-side rule) within the parity
     tolerance (weighted: scaled by the factor a/(1 - a), App. A), the kept
     set outside near ties, bit-exact gathers, sigma of the plain L2 scores
@@ -187,9 +189,19 @@ def test_ex_random_options(orc, case, monkeypatch):
     if running:
         vd.vd_running_sum_init_ex(cache, c["keys"], rs)
     k_new, v_new = st.next(B)
-    vd.vd_append(cache, k_new.view(us + (B, d)).contiguous(), v_new.view(us + (B, d)).contiguous(), B)
-    lens = cache.len.cpu().numpy().copy()
-    pre_k, pre_v = bits(units_view(cache.k)), bits(units_view(cache.v))
+    k_new, v_new = k_new.view(us + (B, d)).contiguous(), v_new.view(us + (B, d)).contiguous()
+    if c["fused"]:
+        # the event's rows: the cached ones, then the new ones at slots len ..
+        lens = cache.len.cpu().numpy().copy() + B
+        pre_k, pre_v = bits(units_view(cache.k)), bits(units_view(cache.v))
+        kn, vn = bits(k_new.view(U, B, d)), bits(v_new.view(U, B, d))
+        for u in range(U):
+            n0 = int(lens[u // per_seq]) - B
+            pre_k[u, n0:n0 + B], pre_v[u, n0:n0 + B] = kn[u], vn[u]
+    else:
+        vd.vd_append(cache, k_new, v_new, B)
+        lens = cache.len.cpu().numpy().copy()
+        pre_k, pre_v = bits(units_view(cache.k)), bits(units_view(cache.v))
     attn = None
     if c["weighted"]:
         g = torch.Generator(device="cuda").manual_seed(c["seed"] % 100003)
@@ -198,8 +210,12 @@ def test_ex_random_options(orc, case, monkeypatch):
     kept = torch.full(us + (N,), -7, dtype=torch.int32, device="cuda")
     scores = torch.full(us + (cap,), float("nan"), device="cuda")
     sigma = torch.full(us, -1.0, device="cuda") if c["disp"] else None
-    vd.vd_evict_block_ex(cache, N, None, B, var, c["mu"], rs if running else None, c["keys"],
-                         attn, kept, scores, sigma)
+    if c["fused"]:
+        vd.vd_append_evict_block_ex(cache, k_new, v_new, B, N, None, var, c["mu"],
+                                    rs if running else None, c["keys"], attn, kept, scores, sigma)
+    else:
+        vd.vd_evict_block_ex(cache, N, None, B, var, c["mu"], rs if running else None,
+                             c["keys"], attn, kept, scores, sigma)
     assert vd.vd_get_device_status() == 0, c
     post_k, post_v = bits(units_view(cache.k)), bits(units_view(cache.v))
     kh, sh = kept.view(U, N).cpu().numpy(), scores.view(U, cap).cpu().numpy()
