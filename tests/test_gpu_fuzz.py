@@ -14,6 +14,8 @@ new length, and the running sum against a from-scratch sum.  Needs a GB300.
 """
 from __future__ import annotations
 
+import os
+
 import numpy as np
 import pytest
 import torch
@@ -26,8 +28,9 @@ from vd_gpu import bits, check_event, new_cache, units_view
 
 pytestmark = pytest.mark.gpu
 HEAD_DIMS = [8, 16, 24, 40, 64, 72, 128, 136, 200, 256]
-N_CASES = 48
-N_MEDIUM = 8  # budgets of 1000-6000 tokens, the batched score paths' head dims
+# case counts (VD_FUZZ_CASES / VD_FUZZ_MEDIUM / VD_FUZZ_EX widen a run)
+N_CASES = int(os.environ.get("VD_FUZZ_CASES", "48"))
+N_MEDIUM = int(os.environ.get("VD_FUZZ_MEDIUM", "8"))  # budgets of 1000-6000 tokens
 
 
 @pytest.fixture(scope="module", autouse=True)
@@ -144,7 +147,7 @@ def test_fused_random_shapes(orc, case, monkeypatch):
             assert torch.max(torch.abs(ref - rs)).item() <= 1e-12 * scale, (c, event)
 
 
-N_EX = 24  # vd_evict_block_ex: key-side rule, attention weights, sigma by-product
+N_EX = int(os.environ.get("VD_FUZZ_EX", "24"))  # the scoring options of vd_evict_block_ex
 
 
 def draw_ex(i):
