@@ -49,6 +49,7 @@ L2_BYTES = 129 * 2 ** 20
 # ran 4-6x slower than from 8 on the same GB300, although each copy alone
 # runs at ~204 GB/s; the buffers are warmed before the timed region
 E2E_POOL = 8
+CLOCK_TAIL_S = 0.3   # untimed read-only load after the timed region while clocks are sampled
 
 
 # ---------------------------------------------------------------------------
@@ -178,7 +179,7 @@ class ClockSampler:
         try:
             self.proc = subprocess.Popen(
                 ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}",
-                 "--format=csv,noheader,nounits", "-lms", "50"],
+                 "--format=csv,noheader,nounits", "-lms", "20"],
                 stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
             self._t = threading.Thread(target=self._read, daemon=True)
             self._t.start()
@@ -189,8 +190,11 @@ class ClockSampler:
         for line in self.proc.stdout:
             self.lines.append((time.time(), line.strip()))
 
-    def mark(self, t0, t1):
-        self.window = (t0, t1)
+    def mark(self, t0, t1, t2=None):
+        """[t0, t1]: the timed region; [t1, t2]: untimed read-only passes over
+        the same cache (clock_tail), so that a timed region shorter than a
+        few sampling periods still has samples under load."""
+        self.window = (t0, t1, t2 if t2 is not None else t1)
 
     def stop(self):
         if self.proc is None:
@@ -205,8 +209,11 @@ class ClockSampler:
         sm, mx, reasons = [], [], set()
         names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
         lines = self.lines
+        timed = None
         if self.window is not None:
-            inside = [ln for ts, ln in lines if self.window[0] <= ts <= self.window[1] + 0.06]
+            t0, t1, t2 = self.window
+            timed = sum(1 for ts, _ in lines if t0 <= ts <= t1 + 0.02)
+            inside = [ln for ts, ln in lines if t0 <= ts <= t2 + 0.02]
             lines = inside if inside else [ln for _, ln in lines[-3:]]
         else:
             lines = [ln for _, ln in lines]
@@ -225,8 +232,13 @@ class ClockSampler:
         if not sm:
             return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"], "samples": 0}
         sm.sort()
-        return {"sm_mhz": sm[len(sm) // 2], "sm_max_mhz": max(mx), "reasons": sorted(reasons),
-                "samples": len(sm)}
+        out = {"sm_mhz": sm[len(sm) // 2], "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+               "samples": len(sm)}
+        if timed is not None:
+            out["samples_in_timed_region"] = timed
+            out["window"] = "timed region + %.2f s of read-only sigma passes over the same cache" % (
+                self.window[2] - self.window[1])
+        return out
 
 
 # ---------------------------------------------------------------------------
@@ -668,6 +680,22 @@ def h2d_rate(w, nbytes, reps=5):
     return nbytes / (times[len(times) // 2] / 1e3) / 1e9
 
 
+def clock_tail(w, seconds):
+    """Keeps the GPU streaming the workload's cache for `seconds` after the
+    timed region, so that a timed region shorter than a few sampling periods
+    (20 ms) still has clock samples under load.  The passes are read-only
+    (vd_score_ex with only the per-unit sigma as output): the cache, its
+    length and the running sum stay as the timed steps left them, for the
+    measurements that follow."""
+    import torch
+    sigma = torch.empty(w.cache.unit_shape(), device=w.cache.k.device)
+    t0 = time.time()
+    while time.time() - t0 < seconds:
+        for _ in range(8):
+            w.vd.vd_score_ex(w.cache, w.vd.VD_SCORE_L2, False, None, sigma)
+        torch.cuda.synchronize()
+
+
 def measure_gpu(w, steps, warmup, device, e2e_steps):
     import torch
     for _ in range(warmup):
@@ -688,7 +716,9 @@ def measure_gpu(w, steps, warmup, device, e2e_steps):
         w.step(kept[i], evs[i])
     stop.record()
     torch.cuda.synchronize()
-    clocks.mark(t_begin, time.time())
+    t_end = time.time()
+    clock_tail(w, CLOCK_TAIL_S)
+    clocks.mark(t_begin, t_end, time.time())
     clk = clocks.stop()
     barrier(device)
     step_ms = start.elapsed_time(stop)

@@ -107,3 +107,46 @@ def test_reference_arm_runs_on_cpu(monkeypatch):
     assert line["impl"] == "reference" and line["value"] > 0 and line["steps"] == 1
     assert line["cpu_baseline"]["kind"] == "oracle" and line["cpu_baseline"]["cores"] >= 1
     assert line["e2e"]["h2d_bytes_per_step"] == 0 and line["higher_is_better"] is True
+
+
+class _DoneProc:
+    """Stands in for the nvidia-smi child process of a ClockSampler."""
+
+    def terminate(self):
+        pass
+
+    def wait(self, timeout=None):
+        return 0
+
+
+def test_clock_sampler_window():
+    """Samples count from the start of the timed region to the end of the
+    untimed run-on; the idle samples before are left out; the timed region's
+    own count is reported; any active slowdown reason is kept."""
+    cs = bench.ClockSampler(0)
+    cs.proc = _DoneProc()
+    row = "{},2070,0x0,Not Active,Not Active,Not Active,{}"
+    cs.lines = [(0.5, row.format(1200, "Not Active")),             # idle, before
+                (1.00, row.format(2070, "Not Active")),            # timed region
+                (1.02, row.format(2070, "Not Active")),
+                (1.10, row.format(2040, "Active")),                # run-on
+                (1.30, row.format(2070, "Not Active")),
+                (2.00, row.format(900, "Not Active"))]             # after
+    cs.mark(0.99, 1.03, 1.31)
+    out = cs.stop()
+    assert out["samples"] == 4
+    assert out["samples_in_timed_region"] == 2
+    assert out["sm_mhz"] == 2070.0 and out["sm_max_mhz"] == 2070.0
+    assert out["reasons"] == ["sw_power_cap"]
+    assert "read-only" in out["window"]
+
+
+def test_clock_sampler_without_samples_in_window():
+    """No sample inside the window: the last three are reported instead."""
+    cs = bench.ClockSampler(0)
+    cs.proc = _DoneProc()
+    row = "2070,2070,0x0,Not Active,Not Active,Not Active,Not Active"
+    cs.lines = [(5.0, row), (5.1, row), (5.2, row), (5.3, row)]
+    cs.mark(1.0, 1.01, 1.02)
+    out = cs.stop()
+    assert out["samples"] == 3 and out["samples_in_timed_region"] == 0
