@@ -143,11 +143,14 @@ def kernel_source_hash() -> str:
     return h.hexdigest()[:16]
 
 
-def ncu_traffic(workload: str, layout: str = "ordered", separate: bool = False):
+def ncu_traffic(workload: str, layout: str = "ordered", separate: bool = False,
+                kernel: str | None = None, units: int | None = None, mu: str | None = None):
     """DRAM bytes per launch of the eviction kernel from the committed ncu
-    summary, if it was taken on the current kernel sources; else None.
-    separate: a prefill step that appends with vd_append first (its eviction
-    then finds the new rows in the cache, partly still in L2)."""
+    summary, if it was taken on the current kernel sources and (where given)
+    for the same kernel instantiation, number of units and mean mode as this
+    run; else None.  separate: a prefill step that appends with vd_append
+    first (its eviction then finds the new rows in the cache, partly still
+    in L2)."""
     path = os.path.join(ROOT, "profiles", "traffic.json")
     try:
         with open(path) as f:
@@ -156,6 +159,9 @@ def ncu_traffic(workload: str, layout: str = "ordered", separate: bool = False):
         e = t[key + (":separate" if separate else "")]
         if e.get("source_hash") != kernel_source_hash():
             return None
+        for field, want in (("kernel", kernel), ("units", units), ("mu", mu)):
+            if want is not None and e.get(field) != want:
+                return None
         return float(e["dram_bytes_per_launch"])
     except Exception:
         return None
@@ -913,6 +919,15 @@ def run_vd(args):
         tok = w.head_tokens_per_step()
         alg, nominal = w.bytes_per_launch(m["moved"])
         achieved = alg / (kern_ms / 1e3) / 1e9
+        kernel = (f"vd::evict_kernel<{variant}, {str(isinstance(w, Decode)).lower()}, "
+                  f"{str(layout == 'holefill').lower()}, "
+                  f"{str(getattr(w, 'fused', False)).lower()}>")
+        traffic = None
+        if not (set(opts) - {"separate_append"}):   # scoring options: never captured
+            traffic = ncu_traffic(name, layout, separate=not getattr(w, "fused", True),
+                                  kernel=kernel, units=w.U,
+                                  mu="running" if (mu if mu_mode is None else mu_mode)
+                                  == vd.VD_MU_RUNNING else "recompute")
         res = {
             "workload": name, "w": w, "m": m, "step_ms": step_ms, "kern_ms": kern_ms,
             "value": tok * ws / (step_ms / 1e3),
@@ -921,11 +936,8 @@ def run_vd(args):
                     "h2d_gbs_alone": m["link_gbs"]},
             "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                          "frac": achieved / peak,
-                         "traffic": ncu_traffic(name, layout, separate=not getattr(w, "fused", True))
-                         if not (set(opts) - {"separate_append"}) else None,
-                         "kernel": f"vd::evict_kernel<{variant}, {str(isinstance(w, Decode)).lower()}, "
-                                   f"{str(layout == 'holefill').lower()}, "
-                                   f"{str(getattr(w, 'fused', False)).lower()}>",
+                         "traffic": traffic,
+                         "kernel": kernel,
                          "algorithmic_bytes_per_launch": alg,
                          "nominal_bytes_per_launch": nominal,
                          "moved_rows_per_launch": m["moved"],

@@ -92,6 +92,13 @@ def test_traffic_is_reported_only_for_the_captured_sources(monkeypatch):
     monkeypatch.setattr(bench, "kernel_source_hash", lambda: t["prefill_wide"]["source_hash"])
     assert bench.ncu_traffic("prefill_wide") == t["prefill_wide"]["dram_bytes_per_launch"]
     assert bench.ncu_traffic("no_such_workload") is None
+    e = t["prefill_wide"]
+    # the same kernel, units and mean mode as the capture, or nothing
+    assert bench.ncu_traffic("prefill_wide", kernel=e["kernel"], units=e["units"],
+                             mu=e["mu"]) == e["dram_bytes_per_launch"]
+    assert bench.ncu_traffic("prefill_wide", units=e["units"] // 2) is None
+    assert bench.ncu_traffic("prefill_wide", kernel=e["kernel"].replace("<0,", "<1,")) is None
+    assert bench.ncu_traffic("prefill_wide", mu="recompute") is None
     monkeypatch.setattr(bench, "kernel_source_hash", lambda: "changed")
     assert bench.ncu_traffic("prefill_wide") is None
 
