@@ -86,12 +86,26 @@ def barrier(device=None):
             dist.barrier()
 
 
+def nvml_id(device_index: int) -> str:
+    """The GPU's id for `nvidia-smi -i`: its UUID, since CUDA and NVML may
+    number the GPUs differently (CUDA_VISIBLE_DEVICES, device order); the
+    CUDA index where torch does not report a UUID."""
+    try:
+        import torch
+        u = str(torch.cuda.get_device_properties(device_index).uuid)
+        if u:
+            return u if u.startswith("GPU-") else "GPU-" + u
+    except Exception:
+        pass
+    return str(device_index)
+
+
 def bind_to_gpu_numa(gpu_index: int):
     """Pins this process to the host CPUs local to the GPU (sysfs local_cpulist
     of its PCI device), so pinned host buffers are allocated on the GPU's own
     NUMA node; returns the CPU list or None."""
     try:
-        bus = subprocess.run(["nvidia-smi", "-i", str(gpu_index), "--query-gpu=pci.bus_id",
+        bus = subprocess.run(["nvidia-smi", "-i", nvml_id(gpu_index), "--query-gpu=pci.bus_id",
                               "--format=csv,noheader"], capture_output=True, text=True,
                              timeout=20).stdout.strip()
         dom, rest = bus.split(":", 1)
@@ -184,7 +198,7 @@ class ClockSampler:
     def start(self):
         try:
             self.proc = subprocess.Popen(
-                ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}",
+                ["nvidia-smi", "-i", nvml_id(self.gpu), f"--query-gpu={self.FIELDS}",
                  "--format=csv,noheader,nounits", "-lms", "20"],
                 stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
             self._t = threading.Thread(target=self._read, daemon=True)
