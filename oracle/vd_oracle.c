@@ -135,10 +135,14 @@ typedef struct {
 } vdo_ranked;
 
 /* Order of Eq. (eviction)'s top-N: higher score first; among equal scores the
- * lower (earlier) cache slot first. */
+ * lower (earlier) cache slot first.  A NaN score (only an invalid input makes
+ * one) ranks below every number, so it is evicted first; NaNs tie among
+ * themselves.  -0 and +0 are equal. */
 static int vdo_rank_cmp(const void* pa, const void* pb) {
   const vdo_ranked* a = (const vdo_ranked*)pa;
   const vdo_ranked* b = (const vdo_ranked*)pb;
+  const int a_nan = isnan(a->score), b_nan = isnan(b->score);
+  if (a_nan != b_nan) return a_nan - b_nan;
   if (a->score > b->score) return -1;
   if (a->score < b->score) return 1;
   return (a->index > b->index) - (a->index < b->index);

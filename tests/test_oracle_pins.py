@@ -127,3 +127,22 @@ def test_weights_outside_unit_interval_give_nan(orc):
     v = pins.gauss_cache(np.random.default_rng(1), 4, 4)
     s = orc.scores_weighted(v, np.array([0.2, 1.0, -0.1, 0.0]), oracle.L2)
     assert np.isnan(s[1]) and np.isnan(s[2]) and s[3] == 0.0 and s[0] > 0
+
+
+def test_nan_ranks_below_zero_and_negative_zero_equals_zero(orc):
+    """Reading where the paper is silent: a NaN score (only an invalid input
+    makes one) is evicted before any number, including a zero score at a
+    higher slot; -0 ties with +0 and the lower slot wins.  Checked against the
+    brute-force rank with NaN mapped below every number."""
+    s = np.array([np.nan, 0.0, -0.0, 3.0, np.nan, 0.0, 2.0])
+    assert list(orc.select_top_n(s, 3)) == [1, 3, 6]
+    assert list(orc.select_top_n(s, 5)) == [1, 2, 3, 5, 6]
+    assert list(orc.select_top_n(s, 6)) == [0, 1, 2, 3, 5, 6]
+    key = np.where(np.isnan(s), -np.inf, s)
+    for N in range(1, len(s)):
+        assert np.array_equal(orc.select_top_n(s, N), pins.brute_force_kept(key, N))
+    # a weight of -0 gives a score of -0, which ranks with the zeros
+    v = pins.gauss_cache(np.random.default_rng(3), 4, 4)
+    w = orc.scores_weighted(v, np.array([0.5, -0.0, 0.0, 1.0]), oracle.L2)
+    assert w[1] == 0.0 and w[2] == 0.0 and np.isnan(w[3])
+    assert list(orc.select_top_n(w, 3)) == [0, 1, 2]
