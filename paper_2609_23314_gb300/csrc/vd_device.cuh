@@ -76,11 +76,15 @@ __device__ __forceinline__ unsigned long long bf16x2_to_f2(uint32_t w) {
   return f2_pack(__uint_as_float(w << 16), __uint_as_float(w & 0xffff0000u));
 }
 
+// 16-byte global load through L2 only.  The "memory" clobber keeps it in
+// program order with the plain C++ stores around it (the hole-fill path
+// writes positions and slot maps between row moves).
 __device__ __forceinline__ uint4 ld_cg16(const void* p) {
   uint4 r;
   asm volatile("ld.global.cg.v4.u32 {%0,%1,%2,%3}, [%4];"
                : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w)
-               : "l"(p));
+               : "l"(p)
+               : "memory");
   return r;
 }
 
@@ -105,6 +109,16 @@ __device__ __forceinline__ uint4 ld_shared16(uint32_t addr) {
                : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w)
                : "r"(addr)
                : "memory");
+  return r;
+}
+
+// 8-byte shared-memory load into a packed fp32 pair.  volatile: issued at
+// each use (a loop-invariant value the compiler would otherwise keep in
+// registers); the data is written before the block barrier that precedes
+// every use, so no memory clobber is needed.
+__device__ __forceinline__ unsigned long long ld_shared_b64(uint32_t addr) {
+  unsigned long long r;
+  asm volatile("ld.shared.b64 %0, [%1];" : "=l"(r) : "r"(addr));
   return r;
 }
 

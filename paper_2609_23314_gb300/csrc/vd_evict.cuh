@@ -8,14 +8,17 @@
 //   1. mean   mean = (1/n) sum_i v_i (Sec. 3.2, Eq. vd) as double-float
 //             (hi + lo) fp32 column sums; the C partials are added in rank
 //             order through distributed shared memory (DSMEM), so every CTA
-//             holds the same mean.  Running-sum mode adds only the appended
-//             rows (spread over the cluster) to the caller's fp64 sum S.
+//             holds the same mean, kept as an fp32 part plus its remainder.
+//             Running-sum mode adds only the appended rows (spread over the
+//             cluster) to the caller's fp64 sum S.
 //   2. score  rows stream through a per-thread ring of asynchronous 16-byte
 //             copies (cp.async, 4 stages in flight); d/8 lanes per row, warp
-//             shuffle reduction of the squared deviation (L2), of the norm
-//             (Norm), or of the normalised difference (Dir, as
-//             1/2 |v/|v| - mean/|mean||^2, which equals 1 - cos without
-//             cancellation).  For d = 64, 128, 256 (L2, Norm) each lane keeps
+//             shuffle reduction of the squared deviation (L2, as
+//             ((v - hi) - lo)^2 against the two-part mean), of the norm
+//             (Norm), or of |w|^2 / (2 |v|^2) with w = v - (|v|/|mean|) mean
+//             (Dir: equals 1 - cos without cancellation).  Every score's
+//             rounding error is relative to the score itself.
+//             For d = 64, 128, 256 (L2, Norm) each lane keeps
 //             a batch of 8 rows' partial sums (packed f32x2 arithmetic) and
 //             the batch is reduced with a transposed butterfly
 //             (score_rows_fast).  Scores become order-preserving uint32 keys.
@@ -138,8 +141,9 @@ struct EvictArgs {
 // cp.async ring, then (block eviction only) this CTA's keys [R] and the
 // unit's perm [capacity] (uint16).
 struct Smem {
-  float mu[256];
-  float muhat[256];
+  float mu[256];    // the mean rounded to fp32 ...
+  float mulo[256];  // ... and its remainder (mean = mu + mulo to ~2^-44 relative),
+                    // pair-transposed: column c at lo_index(c, d / 8)
   float acc_hi[256];  // this CTA's partial column sums (read by peer CTAs)
   float acc_lo[256];
   double snew[256];       // running mode: the running sum plus the appended rows
@@ -155,10 +159,19 @@ struct Smem {
   int best_slot;       // hole-fill decode: the slot of `best`
   int wslot[kWarps];
   int holes;           // hole-fill: evicted slots below N
+  float inv_mnorm;     // Dir: 1 / |mean|
   float disp[4];       // dispersion partials: sum s (hi, lo), sum s^2 (hi, lo)
+  float dsc[4 * kWarps];  // dispersion: per-warp partials (block-private)
 };
 
 __host__ __device__ constexpr size_t align16(size_t x) { return (x + 15) & ~(size_t)15; }
+
+// Slot of column c of the mean's remainder in Smem::mulo (d8 = d / 8 chunks
+// of 8 columns): the pairs (2k, 2k + 1) of every chunk are stored together,
+// pair k of chunk ci at floats 2 * (k * d8 + ci) and + 1.
+__device__ __forceinline__ int lo_index(int c, int d8) {
+  return 2 * (((c & 7) >> 1) * d8 + (c >> 3)) + (c & 1);
+}
 
 // Byte offsets of the variable parts; the host sizes the launch with the same
 // function.  The ring starts on a 128-byte boundary: a warp's 16-byte copies
@@ -228,16 +241,23 @@ __device__ __forceinline__ void stream_rows(int chunk0, int nchunks, int P, int 
 }
 
 // Squared norm of one 16-byte chunk (8 bf16 values) of a row: of v - mean
-// for VAR 0 (m2: the chunk's mean as packed pairs), of v itself for VAR 2.
-template <int VAR>
-__device__ __forceinline__ float chunk_sq(const uint4& q, const unsigned long long (&m2)[4]) {
+// for VAR 0, of v itself for VAR 2.  The chunk's mean arrives as packed
+// pairs of its fp32 part m2 and remainder l2: (x - m2) - l2 is rounded
+// relative to x - mean itself, so the score's error is relative to the
+// score (with the fp32 mean alone it would carry an absolute 2^-24 |mean|).
+template <int VAR, int LPR>
+__device__ __forceinline__ float chunk_sq(const uint4& q, const unsigned long long (&m2)[4],
+                                          uint32_t lo_addr) {
   const uint32_t w[4] = {q.x, q.y, q.z, q.w};
   unsigned long long acc = 0ull;
 #pragma unroll
   for (int k = 0; k < 4; ++k) {
     const unsigned long long x = bf16x2_to_f2(w[k]);
     if (VAR == 0) {
-      const unsigned long long dv = f2_sub(x, m2[k]);
+      // the remainder pair is read from shared memory at each use rather
+      // than held in registers (the kernels sit at their register limit)
+      const unsigned long long l2 = ld_shared_b64(lo_addr + (uint32_t)(k * LPR * 8));
+      const unsigned long long dv = f2_sub(f2_sub(x, m2[k]), l2);
       acc = f2_fma(dv, dv, acc);
     } else {
       acc = f2_fma(x, x, acc);
@@ -256,12 +276,15 @@ __device__ __forceinline__ float chunk_sq(const uint4& q, const unsigned long lo
 // ci % (LPR / kBatch) == 0 call finish(j, s) for the batch's valid rows (j is
 // the row's index in [0, R)).  Same arithmetic per element as the general
 // path; only the order of the fp32 additions differs.
-template <int VAR, int LPR, class Ring, class Finish>
+template <int VAR, int LPR, class Ring, int BATCH, class Finish>
 __device__ __forceinline__ void score_rows_fast(const uint16_t* __restrict__ rows, int R,
-                                                const float* mu, Finish finish, uint32_t ring) {
+                                                const float* mu, const float* mulo,
+                                                Finish finish, uint32_t ring) {
   constexpr int kStages = Ring::kStages, kItems = Ring::kItems;
-  constexpr int kBatch = 8;
-  static_assert(kBatch % kItems == 0 && LPR >= kBatch, "batch shape");
+  constexpr int kBatch = BATCH;
+  constexpr int kLogBatch = kBatch == 8 ? 3 : kBatch == 4 ? 2 : 1;
+  static_assert((1 << kLogBatch) == kBatch && kBatch % kItems == 0 && LPR >= kBatch,
+                "batch shape");
   constexpr int kStagesPerBatch = kBatch / kItems;
   constexpr int kGroups = kThreads / LPR;
   constexpr int kD = LPR * 8;
@@ -271,6 +294,9 @@ __device__ __forceinline__ void score_rows_fast(const uint16_t* __restrict__ row
 #pragma unroll
   for (int k = 0; k < 4; ++k)
     m2[k] = VAR == 0 ? f2_pack(mu[ci * 8 + 2 * k], mu[ci * 8 + 2 * k + 1]) : 0ull;
+  // mulo is in the pair-transposed layout (lo_index): pair k of chunk ci at
+  // float 2 * (k * LPR + ci), so a warp's loads of one pair hit distinct banks
+  const uint32_t lo_addr = smem_addr(mulo) + (uint32_t)ci * 8u;
   const int per_stage = kGroups * kItems;
   const int nst = (R + per_stage - 1) / per_stage;
   const uint32_t my = ring + (uint32_t)tid * 16u;
@@ -301,13 +327,13 @@ __device__ __forceinline__ void score_rows_fast(const uint16_t* __restrict__ row
         const int k = st * kItems + u;
         uint4 q = make_uint4(0u, 0u, 0u, 0u);
         if (g + k * kGroups < R) q = ld_shared16(slot(st % kStages, u));
-        part[sb * kItems + u] = chunk_sq<VAR>(q, m2);
+        part[sb * kItems + u] = chunk_sq<VAR, LPR>(q, m2, lo_addr);
       }
       issue(st + kStages);
     }
     // transposed steps over lane offsets LPR/2, LPR/4, LPR/8
 #pragma unroll
-    for (int j = 0; j < 3; ++j) {
+    for (int j = 0; j < kLogBatch; ++j) {
       const int h = kBatch >> (j + 1), off = LPR >> (j + 1);
       const bool upper = (ci & off) != 0;
 #pragma unroll
@@ -381,11 +407,18 @@ __device__ __forceinline__ void sum_rows(int chunk0, int nchunks, int P, int cou
   merge_columns(hi, lo, P, active, (chunk0 + ci) * 8, S.acc_hi, S.acc_lo);
 }
 
-// Order-preserving key of a non-negative score; NaN ranks lowest.  `bad`
-// reports a NaN or infinite score.
+// Order-preserving key of a score (scores are never negative): a positive
+// score maps to its bit pattern + 1 (+inf to 0x7f800001), +0 and -0 both to
+// 1, and NaN to 0, strictly below every number, so a NaN ranks lowest and
+// never ties with a zero score.  `bad` reports a NaN or infinite score.
 __device__ __forceinline__ uint32_t score_key(float s, bool& bad) {
   bad = !(s == s) || s == __int_as_float(0x7f800000);
-  return (s == s) ? __float_as_uint(s) : 0u;
+  return s > 0.f ? __float_as_uint(s) + 1u : (s == 0.f ? 1u : 0u);
+}
+
+// The score a key came from (+0 for either zero, NaN for key 0).
+__device__ __forceinline__ float key_score(uint32_t key) {
+  return key ? __uint_as_float(key - 1u) : __int_as_float(0x7fc00000);
 }
 
 // Dispersion of the L2 scores over a unit (Sec. 3.1: sigma = std_j s_j):
@@ -875,14 +908,19 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
         sum += rs_own;
         S.snew[tid] = sum;  // phase 5 starts from it
       }
-      S.mu[tid] = (float)(sum / (double)n);
+      const double m = sum / (double)n;
+      const float mh = (float)m;
+      S.mu[tid] = mh;
+      S.mulo[lo_index(tid, d8)] = (float)(m - (double)mh);
     }
     __syncthreads();
     if (VAR == 1) {
       const float m = tid < d ? S.mu[tid] : 0.f;
       const float nrm2 = block_sum_f32(m * m, S.fsh);
-      if (tid < d) S.muhat[tid] = nrm2 > 0.f ? m / sqrtf(nrm2) : 0.f;
-      if (tid == 0) S.mu_zero = !(nrm2 > 0.f);
+      if (tid == 0) {
+        S.mu_zero = !(nrm2 > 0.f);
+        S.inv_mnorm = nrm2 > 0.f ? 1.f / sqrtf(nrm2) : 0.f;
+      }
       __syncthreads();
     }
   }
@@ -897,13 +935,19 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
   {
     const int ci = lane & (lpr - 1);
     const bool active = ci < d8;
-    float m8[8], h8[8];
+    float m8[8];  // this lane's columns of the mean (fp32 part)
 #pragma unroll
-    for (int k = 0; k < 8; ++k) {
-      m8[k] = (VAR == 0 && active) ? S.mu[ci * 8 + k] : 0.f;
-      h8[k] = (VAR == 1 && active) ? S.muhat[ci * 8 + k] : 0.f;
-    }
+    for (int k = 0; k < 8; ++k) m8[k] = (VAR != 2 && active) ? S.mu[ci * 8 + k] : 0.f;
+    // ... and of its remainder, read in pairs at each use (see chunk_sq)
+    const uint32_t lo_addr = smem_addr(S.mulo) + (uint32_t)(active ? ci : 0) * 8u;
+    auto lo_pair = [&](int k, float& l0, float& l1) {
+      const unsigned long long p = ld_shared_b64(lo_addr + (uint32_t)(k * d8 * 8));
+      l0 = __uint_as_float((uint32_t)p);
+      l1 = __uint_as_float((uint32_t)(p >> 32));
+      if (!active) l0 = l1 = 0.f;
+    };
     const bool mu_zero = VAR == 1 && S.mu_zero;
+    const float inv_mnorm = VAR == 1 ? S.inv_mnorm : 0.f;
     const bool weighted = !DECODE && a.weights != nullptr;
     float ds_hi = 0.f, ds_lo = 0.f, dq_hi = 0.f, dq_lo = 0.f;  // dispersion sums
     unsigned long long best = ~0ull;  // (key, tie-break) of this thread's minimum
@@ -942,16 +986,21 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
       }
     };
     bool fast = false;
+    // rows per batch: 4 in the ordered decode kernels, whose other live state
+    // (the running arg-min, the staged-row pointers) leaves no room for 8
+    // rows' partial sums within 64 registers without spilling
+    constexpr int kScoreBatch = DECODE && !HF ? 4 : 8;
     if constexpr (VAR != 1) {  // head dims 64, 128, 256: one 16-byte chunk per lane
       // cache rows [r0, c_end), then (fused append) staging rows [c_end, r1)
       const int c_end = min(r1, max(r0, first_stage));
       auto run = [&](auto lanes) {
         constexpr int LPR = decltype(lanes)::value;
         if (c_end > r0)
-          score_rows_fast<VAR, LPR, Ring>(sb + (size_t)r0 * d, c_end - r0, S.mu, finish_row, ring);
+          score_rows_fast<VAR, LPR, Ring, kScoreBatch>(sb + (size_t)r0 * d, c_end - r0, S.mu, S.mulo,
+                                          finish_row, ring);
         if (r1 > c_end)
-          score_rows_fast<VAR, LPR, Ring>(
-              snu + (size_t)(c_end - first_stage) * d, r1 - c_end, S.mu,
+          score_rows_fast<VAR, LPR, Ring, kScoreBatch>(
+              snu + (size_t)(c_end - first_stage) * d, r1 - c_end, S.mu, S.mulo,
               [&](int j, float s) { finish_row(j + (c_end - r0), s); }, ring);
       };
       fast = true;
@@ -974,9 +1023,13 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
           if (VAR == 0) {
             float acc = 0.f;
 #pragma unroll
-            for (int k = 0; k < 8; ++k) {
-              const float dv = x[k] - m8[k];
-              acc = fmaf(dv, dv, acc);
+            for (int k = 0; k < 8; k += 2) {
+              float l0, l1;
+              lo_pair(k >> 1, l0, l1);
+              const float dv0 = (x[k] - m8[k]) - l0;
+              const float dv1 = (x[k + 1] - m8[k + 1]) - l1;
+              acc = fmaf(dv0, dv0, acc);
+              acc = fmaf(dv1, dv1, acc);
             }
             for (int off = 1; off < lpr; off <<= 1) acc += __shfl_xor_sync(kFull, acc, off);
             s = sqrtf(acc);
@@ -987,27 +1040,34 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
             for (int off = 1; off < lpr; off <<= 1) acc += __shfl_xor_sync(kFull, acc, off);
             s = sqrtf(acc);
           } else {
+            // 1 - cos(v, m) = |w|^2 / (2 |v|^2) with w = v - (|v| / |m|) m:
+            // each w_c is one fused multiply-add of the row and the
+            // double-float mean, rounded relative to w_c itself, so the
+            // score's error stays relative to the score even where v and m
+            // are nearly parallel (1 - cos computed directly would cancel)
             float nv = 0.f;
 #pragma unroll
             for (int k = 0; k < 8; ++k) nv = fmaf(x[k], x[k], nv);
             for (int off = 1; off < lpr; off <<= 1) nv += __shfl_xor_sync(kFull, nv, off);
-            const float inv = nv > 0.f ? 1.f / sqrtf(nv) : 0.f;
+            const float lam = sqrtf(nv) * inv_mnorm;
             float acc = 0.f;
 #pragma unroll
-            for (int k = 0; k < 8; ++k) {
-              const float dv = x[k] * inv - h8[k];
-              acc = fmaf(dv, dv, acc);
+            for (int k = 0; k < 8; k += 2) {
+              float l0, l1;
+              lo_pair(k >> 1, l0, l1);
+              const float w0 = fmaf(-lam, l0, fmaf(-lam, m8[k], x[k]));
+              const float w1 = fmaf(-lam, l1, fmaf(-lam, m8[k + 1], x[k + 1]));
+              acc = fmaf(w0, w0, acc);
+              acc = fmaf(w1, w1, acc);
             }
             for (int off = 1; off < lpr; off <<= 1) acc += __shfl_xor_sync(kFull, acc, off);
-            s = (nv > 0.f && !mu_zero) ? 0.5f * acc : 1.f;
+            s = (nv > 0.f && !mu_zero) ? (0.5f * acc) / nv : 1.f;
           }
           if (in && ci == 0) finish_row(item, s);
         },
         ring);
-    // sigma is defined on the L2 distance (VAR 0), whose scores never read
-    // muhat: it serves as the scratch
     if constexpr (VAR == 0) {
-      if (disp) disp_reduce_cta(ds_hi, ds_lo, dq_hi, dq_lo, S.muhat, S);
+      if (disp) disp_reduce_cta(ds_hi, ds_lo, dq_hi, dq_lo, S.dsc, S);
     }
     if (a.score_only) {
       if (score_split) cluster_wait();
@@ -1084,7 +1144,7 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
       for (int j = tid; j < R; j += kThreads) {
         const float w = wu[r0 + j];
         const float f = (w >= 0.f && w < 1.f) ? w / (1.f - w) : __int_as_float(0x7fc00000);
-        const float sw = __uint_as_float(keys[j]) * f;
+        const float sw = key_score(keys[j]) * f;
         bool bad;
         keys[j] = score_key(sw, bad);
         if (bad) record_status(a.status, kStNonfinite);

@@ -17,3 +17,25 @@ def pytest_configure(config):
 def orc():
     import oracle
     return oracle.load()
+
+
+def pytest_terminal_summary(terminalreporter):
+    """The worst score error each GPU test saw against the oracle, per rule:
+    relative (over scores above 1e-6) and as a fraction of the tolerance."""
+    try:
+        from vd_gpu import WORST
+    except Exception:
+        return
+    if not WORST:
+        return
+    tr = terminalreporter
+    tr.section("worst score error vs the fp64 oracle (tolerance 1e-5 relative)")
+    for (test, rule), (rel, frac, count) in sorted(WORST.items()):
+        tr.write_line(f"{test:<60} {rule:<8} rel {rel:.2e}  of tol {frac:.3f}  ({count} scores)")
+    by_rule = {}
+    for (_, rule), (rel, frac, _) in WORST.items():
+        r = by_rule.setdefault(rule, [0.0, 0.0])
+        r[0], r[1] = max(r[0], rel), max(r[1], frac)
+    for rule, (rel, frac) in sorted(by_rule.items()):
+        tr.write_line(f"overall {rule:<8} worst relative error {rel:.3e}, worst fraction of "
+                      f"the tolerance {frac:.3f}")

@@ -11,7 +11,8 @@ import torch
 import oracle
 import paper_2609_23314_gb300 as vd
 from paper_2609_23314_gb300 import build, workloads as wl
-from vd_gpu import RTOL, bits, near_tie_band, new_cache, score_tolerance, units_view
+from vd_gpu import (RTOL, bits, near_tie_band, new_cache, record_error, score_tolerance,
+                    units_view, weighted_tolerance)
 
 pytestmark = pytest.mark.gpu
 VARS = [oracle.L2, oracle.DIR, oracle.NORM]
@@ -35,13 +36,15 @@ def filled(n_seq, L, H, cap, d, lens, seed, gen="gauss_outlier"):
     return cache
 
 
-def check_scored_event(s_ora, tol, pre_k, pre_v, post_k, post_v, n, N, kept_gpu, scores_gpu):
+def check_scored_event(s_ora, tol, pre_k, pre_v, post_k, post_v, n, N, kept_gpu, scores_gpu,
+                       var=None, tag=""):
     """One unit: GPU scores within tol of the oracle's, the same kept set
     outside near ties, bit-exact gathers of K and V."""
     if n <= N:
         assert np.array_equal(post_v[:n], pre_v[:n]) and np.array_equal(post_k[:n], pre_k[:n])
         return
     err = np.abs(scores_gpu[:n].astype(np.float64) - s_ora)
+    record_error(var, scores_gpu[:n], s_ora, tag, tol)
     assert np.all(err <= tol), f"worst score error {err.max():.3e}"
     kept_ora = orc_select(s_ora, N)
     kg = np.asarray(kept_gpu[:N], np.int64)
@@ -85,10 +88,9 @@ def run_ex(orc, cache, N, B, var, score_keys, attn):
             s_ora = orc.scores_weighted(src, a_h[u, :n], var)
             base = orc.scores(src, var)
             f = a_h[u, :n] / (1.0 - a_h[u, :n])
-            # the weight multiplies the score: its error scales with the factor,
-            # plus one fp32 rounding of the product
-            tol = score_tolerance(var, base, src, orc.mean(src)) * f + 2e-7 * np.abs(s_ora)
-        check_scored_event(s_ora, tol, pre_k[u], pre_v[u], post_k[u], post_v[u], n, N, kh[u], sh[u])
+            tol = weighted_tolerance(var, s_ora, base, src, orc.mean(src), f)
+        check_scored_event(s_ora, tol, pre_k[u], pre_v[u], post_k[u], post_v[u], n, N, kh[u], sh[u],
+                           var, ("_k" if score_keys else "") + ("_w" if a_h is not None else ""))
 
 
 @pytest.mark.parametrize("var", VARS, ids=VAR_IDS)
@@ -110,6 +112,39 @@ def test_attention_weighted_eviction(orc, var, cluster, monkeypatch):
     attn = torch.rand(cache.unit_shape() + (N + B,), generator=g, device="cuda") * 0.9
     attn[..., ::17] = 0.0                     # tokens with no attention score 0
     run_ex(orc, cache, N, B, var, False, attn)
+
+
+@pytest.mark.parametrize("var", VARS, ids=VAR_IDS)
+@pytest.mark.parametrize("cluster", [1, 2])
+def test_negative_zero_weight_and_nan_rank(orc, var, cluster, monkeypatch):
+    """A weight of -0 gives the score -0, which ranks with the zero scores
+    (ties to the lower slot), and a NaN score (a weight of 1, reported as
+    VD_ERR_NONFINITE) ranks below every zero score, so it is evicted first:
+    the kept set equals the oracle's, which orders NaN last."""
+    monkeypatch.setenv("VD_CLUSTER_SIZE", str(cluster))
+    d, n, N = 64, 120, 95
+    cache = filled(1, 1, 2, n, d, [n], seed=31 + cluster)
+    attn = torch.full(cache.unit_shape() + (n,), 0.3, device="cuda")
+    attn[..., :40] = 0.0
+    attn[..., 0:40:2] = -0.0                  # 20 tokens weighted -0
+    attn[..., 1:40:4] = 1.0                   # 10 tokens with a NaN score
+    pre_v = bits(units_view(cache.v))
+    kept = torch.full(cache.unit_shape() + (N,), -7, dtype=torch.int32, device="cuda")
+    scores = torch.full(cache.unit_shape() + (n,), float("nan"), device="cuda")
+    vd.vd_evict_block_ex(cache, N, variant=var, attn=attn, kept_idx_out=kept, scores_out=scores)
+    assert vd.vd_get_device_status() == 4     # VD_ERR_NONFINITE: the NaN scores
+    a_h = attn.view(2, n).cpu().numpy().astype(np.float64)
+    assert np.signbit(a_h[0, 0]) and a_h[0, 0] == 0.0
+    kh = kept.view(2, N).cpu().numpy()
+    sh = scores.view(2, n).cpu().numpy()
+    for u in range(2):
+        s_ora = orc.scores_weighted(pre_v[u, :n], a_h[u], var)
+        want = orc.select_top_n(s_ora, N)
+        assert np.array_equal(kh[u], want), (u, np.setxor1d(kh[u], want))
+        assert not np.any(np.isin(np.arange(1, 40, 4), kh[u]))   # every NaN evicted
+        # the zero-weighted tokens report a zero score, the NaN ones NaN
+        assert np.all(sh[u, :40][np.isnan(s_ora[:40])] != sh[u, :40][np.isnan(s_ora[:40])])
+        assert np.all(sh[u, 0:40:2] == 0.0)
 
 
 def test_uniform_attention_keeps_the_valuediff_set(orc):
@@ -179,6 +214,7 @@ def test_score_ex_running_mean(orc, keys, var, cluster, monkeypatch):
             s_ora = orc.scores(src[u, :n], var)
             tol = score_tolerance(var, s_ora, src[u, :n], orc.mean(src[u, :n]))
             err = np.abs(sh[u, :n].astype(np.float64) - s_ora)
+            record_error(var, sh[u, :n], s_ora, "_k" if keys else "", tol)
             assert np.all(err <= tol), (stage, u, float(err.max()))
             assert np.all(np.isnan(sh[u, n:]))
             if sig is not None:
@@ -276,7 +312,7 @@ def test_key_side_running_mean(orc, var, cluster, monkeypatch):
             s_ora = orc.scores(pre_k[u, :n], var)
             tol = score_tolerance(var, s_ora, pre_k[u, :n], orc.mean(pre_k[u, :n]))
             check_scored_event(s_ora, tol, pre_k[u], pre_v[u], post_k[u], post_v[u], n, N,
-                               kh[u], sh[u])
+                               kh[u], sh[u], var, "_k")
         ref = torch.zeros_like(rs)
         vd.vd_running_sum_init_ex(cache, True, ref)
         scale = units_view(cache.k).float().abs().sum(dim=1).max().item()

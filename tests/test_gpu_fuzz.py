@@ -176,7 +176,7 @@ def test_ex_random_options(orc, case, monkeypatch):
     set outside near ties, bit-exact gathers, sigma of the plain L2 scores
     for the units that evicted, and the running sum of the scored tensor."""
     import test_gpu_extensions as tx
-    from vd_gpu import score_tolerance
+    from vd_gpu import score_tolerance, weighted_tolerance
     tx._ORC = orc
     c = draw_ex(case)
     if c["cluster"]:
@@ -239,10 +239,9 @@ def test_ex_random_options(orc, case, monkeypatch):
         else:
             s_ora = orc.scores_weighted(src, a_h[u, :n], var)
             f = a_h[u, :n] / (1.0 - a_h[u, :n])
-            tol = (score_tolerance(var, orc.scores(src, var), src, orc.mean(src)) * f
-                   + 2e-7 * np.abs(s_ora))
+            tol = weighted_tolerance(var, s_ora, orc.scores(src, var), src, orc.mean(src), f)
         tx.check_scored_event(s_ora, tol, pre_k[u], pre_v[u], post_k[u], post_v[u], n, N, kh[u],
-                              sh[u])
+                              sh[u], var, ("_k" if c["keys"] else "") + ("_w" if a_h is not None else ""))
         if sg is not None:
             want = orc.dispersion(src)
             assert abs(sg[u] - want) <= 1e-5 * want + 1e-6, (c, u, sg[u], want)

@@ -10,9 +10,10 @@ import numpy as np
 import pytest
 import torch
 
+import oracle
 import paper_2609_23314_gb300 as vd
 from paper_2609_23314_gb300 import build, workloads as wl
-from vd_gpu import bits, near_tie_band, new_cache, units_view
+from vd_gpu import bits, near_tie_band, new_cache, record_error, score_tolerance, units_view
 
 pytestmark = pytest.mark.gpu
 VARIANTS = [vd.VD_SCORE_L2, vd.VD_SCORE_DIR, vd.VD_SCORE_NORM]
@@ -55,25 +56,20 @@ def evict(cache, N, var):
 @pytest.mark.parametrize("factor", [2.0, 0.5])
 def test_positive_homogeneity(var, factor):
     """V -> a V with a a power of two (exact in bf16 and in every fp32 step):
-    L2 and Norm scores scale by a bit for bit, Dir scores do not change; the
+    L2 and Norm scores scale by a bit for bit, Dir scores do not change (bit
+    for bit too: |v|, |m| and w = v - (|v|/|m|) m all scale exactly); the
     kept set does not change."""
     n, N = 640, 500
     c1 = filled(n, 128, seed=11)
     c2 = vd.Cache(c1.k.clone(), (c1.v.float() * factor).to(torch.bfloat16), c1.len.clone())
     s1, s2 = scores_of(c1, var)[:, :n], scores_of(c2, var)[:, :n]
     if var == vd.VD_SCORE_DIR:
-        assert torch.max(torch.abs(s2 - s1)).item() <= 1e-6
+        assert torch.equal(s2, s1)
     else:
         assert torch.equal(s2, s1 * factor)
     k1, _ = evict(c1, N, var)
     k2, _ = evict(c2, N, var)
-    if var == vd.VD_SCORE_DIR:
-        band = [near_tie_band(s1[u].double().cpu().numpy(), N) for u in range(c1.units)]
-        for u in range(c1.units):
-            diff = np.setxor1d(k1[u], k2[u])
-            assert np.all(band[u][diff])
-    else:
-        assert np.array_equal(k1, k2)
+    assert np.array_equal(k1, k2)
 
 
 @pytest.mark.parametrize("var", VARIANTS, ids=VAR_IDS)
@@ -88,7 +84,9 @@ def test_permutation_equivariance(var):
     s1 = scores_of(c1, var)[:, :n].double().cpu().numpy()
     s2 = scores_of(c2, var)[:, :n].double().cpu().numpy()
     p = perm.numpy()
-    assert np.all(np.abs(s2 - s1[:, p]) <= 1e-6 * np.abs(s1[:, p]) + 1e-7)
+    # the mean is summed in another order: it may differ in its last bits
+    # (relative 1e-12 of the data), which moves a score by about that much
+    assert np.all(np.abs(s2 - s1[:, p]) <= 1e-6 * np.abs(s1[:, p]) + 1e-9)
     k1, _ = evict(c1, N, var)
     k2, _ = evict(c2, N, var)
     for u in range(units):
@@ -135,12 +133,14 @@ def test_scores_equal_the_uniform_attention_disturbance():
     cache = filled(n, d, seed=19, units=units)
     s_gpu = scores_of(cache, vd.VD_SCORE_L2)[:, :n].double().cpu().numpy()
     vals = units_view(cache.v)[:, :n].double().cpu().numpy()
+    rows = bits(units_view(cache.v)[:, :n])
     for u in range(units):
         v = vals[u]
         o = v.mean(axis=0)
         disturb = np.array([(n - 1) * np.linalg.norm(o - np.delete(v, j, axis=0).mean(axis=0))
                             for j in range(n)])
-        tol = 1e-5 * disturb + 2e-6 * (np.linalg.norm(v, axis=1) + np.linalg.norm(o))
+        tol = score_tolerance(oracle.L2, disturb, rows[u], o)
+        record_error(oracle.L2, s_gpu[u], disturb, tol=tol)
         assert np.all(np.abs(s_gpu[u] - disturb) <= tol)
         top_gpu = np.sort(np.argsort(-s_gpu[u], kind="stable")[:N])
         top_bf = np.sort(np.argsort(-disturb, kind="stable")[:N])

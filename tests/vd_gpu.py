@@ -3,17 +3,22 @@ bf16 bit patterns, and compare one eviction event of the CUDA path with the
 fp64 oracle fed the same pre-eviction bytes (step-locked).
 
 Acceptance (per event, per unit):
-* scores: |s_gpu - s_ora| <= 1e-5 s_ora + atol, where atol is the fp32
-  rounding floor of the GPU's arithmetic: 2e-6 (|v_j| + |mean|) for L2 (the
-  squared deviation is a sum of d fp32 terms of size up to (|v_j|+|mean|)^2),
-  1e-6 for Dir (a difference of unit vectors) and 0 for Norm;
+* scores: |s_gpu - s_ora| <= 1e-5 s_ora + atol (the relative tolerance the
+  method's definition is checked at), where atol only covers the accuracy of
+  the mean itself (~1e-11 of the data's scale) and, for Dir, a 1.8e-12
+  floor (score_tolerance derives both);
 * kept sets: identical, except for tokens whose oracle score lies within
   1e-5 s_(N) of the N-th largest oracle score s_(N) (near ties that fp32
   rounding may order either way);
 * compacted K and V: bit-identical to the pre-eviction rows at the GPU's kept
   indices, which are strictly ascending; the length becomes N exactly.
+
+Every score comparison also records the worst relative error it saw, per test
+and rule (``record_error``); the session prints the table at the end.
 """
 from __future__ import annotations
+
+import os
 
 import numpy as np
 import torch
@@ -22,6 +27,37 @@ import oracle
 import paper_2609_23314_gb300 as vd
 
 RTOL = 1e-5
+# Relative accuracy of the kernel's mean (double-float column sums, fp64
+# division, an fp32 part plus an fp32 remainder) with respect to the mean of
+# |v|: the same 1e-12 the running-sum checks hold the sums to.
+MEAN_RTOL = 1e-12
+VAR_NAMES = {oracle.L2: "l2", oracle.DIR: "dir", oracle.NORM: "norm"}
+# Dir: the second-order effect of a 32-ulp error in |v| / |mean| (below)
+DIR_RADIAL_FLOOR = 0.5 * (32 * 2.0 ** -24) ** 2
+
+# (test, rule) -> [worst |ds| / s over scores > 1e-6, worst |ds| / tolerance, count]
+WORST: dict = {}
+
+
+def record_error(var, s_gpu, s_ora, tag: str = "", tol=None):
+    """Tracks, for the session summary, the worst relative score error (over
+    scores above 1e-6, where the relative tolerance is the one that binds)
+    and the worst error as a fraction of the tolerance (1.0 would fail)."""
+    test = os.environ.get("PYTEST_CURRENT_TEST", "?").split(" ")[0].split("::")[-1]
+    key = (test, VAR_NAMES.get(var, str(var)) + tag)
+    s_ora = np.asarray(s_ora, np.float64)
+    err = np.abs(np.asarray(s_gpu, np.float64) - s_ora)
+    big = s_ora > 1e-6
+    rel = float(np.max(err[big] / s_ora[big])) if np.any(big) else 0.0
+    frac = 0.0
+    if tol is not None:
+        t = np.broadcast_to(np.asarray(tol, np.float64), s_ora.shape)
+        ok = t > 0
+        frac = float(np.max(err[ok] / t[ok])) if np.any(ok) else 0.0
+    w = WORST.setdefault(key, [0.0, 0.0, 0])
+    w[0] = max(w[0], rel)
+    w[1] = max(w[1], frac)
+    w[2] += int(s_ora.size)
 
 
 def bits(t: torch.Tensor) -> np.ndarray:
@@ -39,12 +75,46 @@ def units_view(t: torch.Tensor) -> torch.Tensor:
 
 
 def score_tolerance(var, s_ora, v_rows, mu):
+    """Allowed |s_gpu - s_ora| per row: RTOL * s_ora plus an absolute term
+    that covers only the error of the kernel's mean.
+
+    Every rounding the kernel does after the mean is relative to the score
+    itself: the mean enters as an fp32 part plus its fp32 remainder, so
+    L2's deviation (v - hi) - lo is rounded relative to v - mean; the squares
+    and the d-term sums (fp32, at most ~12 levels deep) and the square root
+    add a few 2^-24 relative; Dir's w = v - (|v|/|m|) m is one fused
+    multiply-add per element against the same two-part mean, its radial error
+    (from |v| and |m|) changes the score relatively, and the final division
+    by |v|^2 is one more rounding.  Worst case well under 1e-5 (about 50
+    ulp for Dir, 10 for L2; observed far less).
+
+    What is not relative: the mean's own error dm, |dm| <= MEAN_RTOL * mean|v|
+    per coordinate.  It moves an L2 score by at most |dm| and a Dir score by
+    at most sqrt(2 s) |dm| / |m|.  And for Dir, the second-order part of the
+    radial error: with |v|/|m| off by a relative delta, |w|^2 gains
+    |v|^2 delta^2 on top of the first-order (relative) change, so a row
+    parallel to the mean (s = 0) scores delta^2 / 2.  delta is at most ~32
+    ulp (|v| and |m| from fp32 sums, two square roots, a product), a floor of
+    0.5 (32 * 2^-24)^2 = 1.8e-12.  Norm reads no mean: purely relative."""
+    s_ora = np.asarray(s_ora, np.float64)
+    if var == oracle.NORM:
+        return RTOL * s_ora
+    vals = oracle.bits_to_float(v_rows)
+    dm = MEAN_RTOL * np.linalg.norm(np.abs(vals).mean(axis=0))
     if var == oracle.L2:
-        vn = np.linalg.norm(oracle.bits_to_float(v_rows), axis=1)
-        return RTOL * s_ora + 2e-6 * (vn + np.linalg.norm(mu))
-    if var == oracle.DIR:
-        return RTOL * s_ora + 1e-6
-    return RTOL * s_ora
+        return RTOL * s_ora + dm
+    mn = np.linalg.norm(mu)
+    first = np.sqrt(2.0 * np.maximum(s_ora, 0.0)) * dm / mn if mn > 0 else 0.0
+    return RTOL * s_ora + first + DIR_RADIAL_FLOOR
+
+
+def weighted_tolerance(var, s_weighted, base, v_rows, mu, f):
+    """The attention-weighted score a/(1 - a) * s (App. A): the factor and
+    the product add three fp32 roundings (relative); the mean's absolute
+    term scales with the factor."""
+    s_weighted = np.asarray(s_weighted, np.float64)
+    return RTOL * np.abs(s_weighted) + (score_tolerance(var, base, v_rows, mu)
+                                        - RTOL * np.asarray(base, np.float64)) * f
 
 
 def check_scores(orc, var, pre_v, s_gpu):
@@ -52,6 +122,7 @@ def check_scores(orc, var, pre_v, s_gpu):
     mu = orc.mean(pre_v)
     tol = score_tolerance(var, s_ora, pre_v, mu)
     err = np.abs(s_gpu.astype(np.float64) - s_ora)
+    record_error(var, s_gpu, s_ora, tol=tol)
     bad = np.flatnonzero(err > tol)
     assert bad.size == 0, (f"{bad.size} scores out of tolerance; worst rel "
                            f"{np.max(err / np.maximum(s_ora, 1e-30)):.3e} at {bad[:5]}")
