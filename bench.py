@@ -43,6 +43,7 @@ if ROOT not in sys.path:
 METRIC = "cache tokens scored+compacted/s; HBM GB/s as % of GB300 peak per eviction"
 UNIT = "head-tokens/s"
 FALLBACK_HBM_GBS = 6800.0
+NOMINAL_HBM_GBS = 7900.0   # GB300 HBM3e, nominal (context and the strict fraction)
 L2_BYTES = 129 * 2 ** 20
 # pinned host staging buffers the e2e run cycles through, as a caller's
 # staging pool would: copies from 50 distinct 88 MB pinned blocks (4.4 GB)
@@ -403,6 +404,8 @@ class Prefill:
             extra += self.U * n * 4          # the attention weights
         if self.holefill:
             extra += moved_rows_total * 4 + self.U * self.B * 4
+        self.breakdown = {"scored_rows_read": v_read, "moved_rows_rw": move, "other": extra}
+        if self.holefill:
             return v_read + move + extra, v_read + self.U * self.B * d * 2 * 2 * 2 + extra
         return v_read + move + extra, v_read + self.U * self.N * d * 2 * 2 * 2 + extra
 
@@ -564,6 +567,8 @@ class Decode:
         extra = self.U * d * 8 * 2 if self.mu else 0
         if self.holefill:
             extra += self.U * self.N * 4 + moved_rows_total * 4
+        self.breakdown = {"scored_rows_read": v_read, "moved_rows_rw": move, "other": extra}
+        if self.holefill:
             return v_read + move + extra, v_read + self.U * d * 2 * 2 * 2 + extra
         return v_read + move + extra, v_read + self.U * self.N * d * 2 * 2 * 2 + extra
 
@@ -610,6 +615,86 @@ class Decode:
         return kk, vv, self.N + 1, self.N
 
 
+class RatioDecode(Decode):
+    """Ratio-budget generation (the last `n_steps` tokens of the workload's
+    generation): every step appends one token and evicts to the budget
+    N_t = floor(L_t / 4) of the tokens processed so far, passed per sequence
+    through N_dev.  The budget grows by one every fourth token, so three steps
+    in four evict one row and the fourth only appends.  Steps past n_steps
+    keep the final budget (every step evicts)."""
+
+    def __init__(self, name, cfg, device, seed, mu, variant, n_steps=64, layout="ordered",
+                 separate_append=False):
+        from paper_2609_23314_gb300 import workloads as wl
+        import torch
+        total = cfg["prompt"] + cfg["gen_tokens"]
+        n_steps = max(4, min(n_steps, cfg["gen_tokens"]))
+        self.L0 = total - n_steps + 1                  # tokens processed after the first step
+        self.N_start = wl.budget_at(cfg, self.L0 - 1)  # the cache length before it
+        cfg = dict(cfg, N=wl.budget_at(cfg, total))    # capacity N + 1 at the final budget
+        super().__init__(name, cfg, device, seed, mu, variant, n_tokens=n_steps, layout=layout,
+                         separate_append=separate_append)
+        self.cache.len.fill_(self.N_start)
+        if mu == self.vd.VD_MU_RUNNING:
+            self.rs.zero_()
+            self.vd.vd_running_sum_init(self.cache, self.rs)
+        self.budget = [wl.budget_at(cfg, self.L0 + i) for i in range(n_steps)]
+        self.N_dev = torch.tensor(self.budget, dtype=torch.int32, device=device).view(
+            -1, 1).repeat(1, cfg["n_seq"]).contiguous()
+        self.length = self.N_start     # host copy of every sequence's length
+        self.record = []               # (n, N_t) of the steps measure_gpu times
+        self.recording = False
+
+    def _budget(self):
+        return min(self.i - 1, len(self.budget) - 1)
+
+    def evict(self, evicted=None, kept=None, scores=None):
+        j = self._budget()
+        Nt = self.budget[j]
+        n = self.length + 1
+        self.length = min(n, Nt)
+        if self.recording:
+            self.record.append((n, Nt))
+        k, v = self.pending if self.fused else (None, None)
+        if self.fused:
+            self.vd.vd_append_evict_decode(self.cache, k, v, self.N, self.N_dev[j], self.variant,
+                                           self.mu, self.rs if self.mu else None, evicted, kept,
+                                           scores)
+        else:
+            self.vd.vd_evict_decode(self.cache, self.N, self.N_dev[j], self.variant, self.mu,
+                                    self.rs if self.mu else None, evicted, kept, scores)
+
+    def head_tokens_per_step(self):
+        """Head-tokens scored per timed step: the cached rows of the steps
+        that evicted (a step at the budget only appends)."""
+        rec = self.record or [(self.N + 1, self.N)]
+        return self.U * sum(n for n, Nt in rec if n > Nt) / len(rec)
+
+    def moved_rows(self, evicted_list):
+        rec = self.record or []
+        total = 0
+        for e, (n, Nt) in zip(evicted_list, rec):
+            e = e.long()
+            total += int(self.torch.where(e >= 0, Nt - e, 0).sum().item())
+        return total / max(1, len(evicted_list))
+
+    def bytes_per_launch(self, moved_rows_total):
+        """Per launch, averaged over the timed steps: V read once on the steps
+        that evict, the moved rows, the running sum, and on the steps that only
+        append, the new K and V rows copied in (read and written)."""
+        rec = self.record or [(self.N + 1, self.N)]
+        d = self.d
+        ev = [(n, Nt) for n, Nt in rec if n > Nt]
+        v_read = self.U * d * 2 * sum(n for n, _ in ev) / len(rec)
+        copy_in = self.U * d * 2 * 2 * 2 * (len(rec) - len(ev)) / len(rec)
+        move = moved_rows_total * d * 2 * 2 * 2
+        extra = self.U * d * 8 * 2 if self.mu else 0
+        nominal = v_read + self.U * d * 2 * 2 * 2 * sum(Nt for _, Nt in ev) / len(rec)
+        self.breakdown = {"scored_rows_read": v_read, "moved_rows_rw": move,
+                          "other": copy_in + extra}
+        return v_read + move + copy_in + extra, nominal + copy_in + extra
+
+
 def make_workload(name, device, seed, mu, variant, n_seq=None, events=8, layout="ordered",
                   **opts):
     """`events` = warm-up + timed steps: that many distinct blocks / tokens are
@@ -625,12 +710,9 @@ def make_workload(name, device, seed, mu, variant, n_seq=None, events=8, layout=
     if cfg["kind"] == "decode":
         pool = max(8, min(events, cfg["steps"]))
         return Decode(name, cfg, device, seed, mu, variant, n_tokens=pool, layout=layout, **opts)
-    # ratio budget: its largest event is a decode step at N = 25% of the final length
-    cfg = dict(cfg)
-    total = cfg["prompt"] + cfg["gen_tokens"]
-    cfg["N"] = wl.budget_at(cfg, total)
-    pool = max(8, min(events, cfg["gen_tokens"]))
-    return Decode(name, cfg, device, seed, mu, variant, n_tokens=pool, layout=layout, **opts)
+    # ratio budget: the last `events` steps of the generation, budgets growing
+    return RatioDecode(name, cfg, device, seed, mu, variant, n_steps=max(8, events),
+                       layout=layout, **opts)
 
 
 # ---------------------------------------------------------------------------
@@ -731,10 +813,12 @@ def measure_gpu(w, steps, warmup, device, e2e_steps):
     clocks.start()
     time.sleep(0.5)
     t_begin = time.time()
+    w.recording = True
     start.record()
     for i in range(steps):
         w.step(kept[i], evs[i])
     stop.record()
+    w.recording = False
     torch.cuda.synchronize()
     t_end = time.time()
     clock_tail(w, CLOCK_TAIL_S)
@@ -880,19 +964,87 @@ def cpu_baseline(w, budget_s=2.0, max_units=64):
                       f"single thread: {u1} units x 1 event"}
 
 
-def cpu_model():
-    """The host CPU's model name (x86 'model name', or the Arm part and
-    implementer from /proc/cpuinfo)."""
-    try:
-        with open("/proc/cpuinfo") as f:
-            info = f.read()
-    except OSError:
-        return "unknown"
-    for key in ("model name", "Model", "CPU part"):
-        for line in info.splitlines():
-            if line.startswith(key) and ":" in line:
-                return line.split(":", 1)[1].strip()
-    return "unknown"
+# Arm Ltd. (implementer 0x41) part numbers of server cores, for hosts whose
+# /proc/cpuinfo names no model (Grace reports part 0xd4f)
+ARM_PARTS = {"0xd0c": "Arm Neoverse N1", "0xd40": "Arm Neoverse V1", "0xd49": "Arm Neoverse N2",
+             "0xd4f": "Arm Neoverse V2", "0xd8e": "Arm Neoverse N3", "0xd84": "Arm Neoverse V3"}
+
+
+def cpu_model(cpuinfo: str | None = None):
+    """The host CPU's model name: x86 'model name', else the Arm core named
+    from its implementer and part number in /proc/cpuinfo."""
+    if cpuinfo is None:
+        try:
+            with open("/proc/cpuinfo") as f:
+                cpuinfo = f.read()
+        except OSError:
+            return "unknown"
+    fields = {}
+    for line in cpuinfo.splitlines():
+        if ":" in line:
+            k, v = line.split(":", 1)
+            fields.setdefault(k.strip(), v.strip())
+    for key in ("model name", "Model"):
+        if fields.get(key):
+            return fields[key]
+    part, impl = fields.get("CPU part", "").lower(), fields.get("CPU implementer", "").lower()
+    if impl == "0x41" and part in ARM_PARTS:
+        return f"{ARM_PARTS[part]} (part {part})"
+    return f"part {part}, implementer {impl}" if part else "unknown"
+
+
+def read_peak(device, gib=4, reps=6):
+    """A read-only streaming rate measured in this run (GB/s): torch's sum of
+    a bf16 tensor larger than L2, best of `reps`.  The copy peak of
+    MEASURED_PEAKS.json counts a read and a write per byte moved; kernels
+    that mostly read (the score passes, decode) can exceed it, so every
+    fraction is also reported against the larger of this and the nominal
+    HBM3e rate."""
+    import torch
+    x = torch.ones(gib * 2 ** 30 // 2, dtype=torch.bfloat16, device=device)
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    best = float("inf")
+    for _ in range(reps):
+        torch.cuda.synchronize()
+        a.record()
+        x.sum(dtype=torch.float32)
+        b.record()
+        torch.cuda.synchronize()
+        best = min(best, a.elapsed_time(b))
+    del x
+    torch.cuda.empty_cache()
+    return gib * 2 ** 30 / (best / 1e3) / 1e9
+
+
+def stricter(roofline, read_gbs):
+    """Adds the fractions against the same-run read-only peak and the nominal
+    HBM3e rate, the strictest of the three, and a flag when the copy-peak
+    fraction exceeds 1 (the kernel reads more than it writes, or finds part of
+    its input in L2)."""
+    a = roofline["achieved"]
+    roofline["frac_of_read_peak"] = a / read_gbs if read_gbs else None
+    roofline["frac_of_nominal"] = a / NOMINAL_HBM_GBS
+    roofline["frac_strict"] = a / max(roofline["peak"], read_gbs or 0.0, NOMINAL_HBM_GBS)
+    roofline["above_copy_peak"] = roofline["frac"] > 1.0
+    return roofline
+
+
+def workload_config(name, cfg, mu_name, variant, layout, fused, decode):
+    """The `config` object of a measurement (both arms print the same one)."""
+    from paper_2609_23314_gb300 import workloads as wl
+    cap = (cfg["N"] + cfg["B"]) if cfg["kind"] == "prefill" else None
+    if cfg["kind"] == "decode":
+        cap = cfg["N"] + 1
+    if cfg["kind"] == "ratio":
+        cap = wl.budget_at(cfg, cfg["prompt"] + cfg["gen_tokens"]) + 1
+    cache_gib = wl.units_of(cfg) * cap * cfg["head_dim"] * 4 / 2 ** 30
+    return {"workload": name, **{k: cfg[k] for k in cfg if k not in ("index", "kind")},
+            "mu": mu_name, "variant": variant, "layout": layout,
+            "append": (("fused into the eviction (vd_append_evict_decode)" if decode else
+                        "fused into the eviction (vd_append_evict_block)")
+                       if fused else "vd_append, then the eviction"),
+            "l2": f"inputs larger than L2: cache {cache_gib:.2f} GiB of K+V, touched every step",
+            "storage": "bf16"}
 
 
 def run_vd(args):
@@ -915,6 +1067,7 @@ def run_vd(args):
     mu = vd.VD_MU_RUNNING if args.mu == "running" else vd.VD_MU_RECOMPUTE
     variant = vd.VARIANTS[args.variant]
     peak, peak_src = hbm_peak()
+    read_gbs = max_over_ranks(-read_peak(device), device) * -1.0   # the lowest over ranks
     from paper_2609_23314_gb300 import workloads as wl
 
     def one(name, steps, layout="ordered", mu_mode=None, **opts):
@@ -923,57 +1076,70 @@ def run_vd(args):
             cfg["n_seq"] = args.n_seq
         if args.separate_append:
             opts = dict(opts, separate_append=True)
-        w = make_workload(name, device, rank_seed(wl.BASE_SEED + cfg["index"], rank),
-                          mu if mu_mode is None else mu_mode, variant, args.n_seq,
-                          events=args.warmup + steps, layout=layout, **opts)
-        m = measure_gpu(w, steps, args.warmup, device, min(steps, args.e2e_steps))
+        mm = mu if mu_mode is None else mu_mode
+        e2e_steps = min(steps, args.e2e_steps)
+        w = make_workload(name, device, rank_seed(wl.BASE_SEED + cfg["index"], rank), mm,
+                          variant, args.n_seq, events=args.warmup + steps + e2e_steps + 4,
+                          layout=layout, **opts)
+        m = measure_gpu(w, steps, args.warmup, device, e2e_steps)
         step_ms = max_over_ranks(m["step_ms"], device) / steps
         kern_ms = max_over_ranks(m["kern_ms"], device)
-        e2e_ms = max_over_ranks(m["e2e_ms"], device) / min(steps, args.e2e_steps)
+        e2e_ms = max_over_ranks(m["e2e_ms"], device) / e2e_steps
         tok = w.head_tokens_per_step()
         alg, nominal = w.bytes_per_launch(m["moved"])
         achieved = alg / (kern_ms / 1e3) / 1e9
         kernel = (f"vd::evict_kernel<{variant}, {str(isinstance(w, Decode)).lower()}, "
                   f"{str(layout == 'holefill').lower()}, "
                   f"{str(getattr(w, 'fused', False)).lower()}>")
+        mu_name = "running" if mm == vd.VD_MU_RUNNING else "recompute"
         traffic = None
         if not (set(opts) - {"separate_append"}):   # scoring options: never captured
             traffic = ncu_traffic(name, layout, separate=not getattr(w, "fused", True),
-                                  kernel=kernel, units=w.U,
-                                  mu="running" if (mu if mu_mode is None else mu_mode)
-                                  == vd.VD_MU_RUNNING else "recompute")
+                                  kernel=kernel, units=w.U, mu=mu_name)
         res = {
             "workload": name, "w": w, "m": m, "step_ms": step_ms, "kern_ms": kern_ms,
             "value": tok * ws / (step_ms / 1e3),
             "e2e": {"value": tok * ws / (e2e_ms / 1e3), "unit": UNIT,
                     "h2d_bytes_per_step": m["bi"], "d2h_bytes_per_step": m["bo"],
                     "h2d_gbs_alone": m["link_gbs"]},
-            "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
-                         "frac": achieved / peak,
-                         "traffic": traffic,
-                         "kernel": kernel,
-                         "algorithmic_bytes_per_launch": alg,
-                         "nominal_bytes_per_launch": nominal,
-                         "moved_rows_per_launch": m["moved"],
-                         "kernel_ms": kern_ms, "peak_source": peak_src + ", of measured"
-                         if "measured" in peak_src else peak_src},
-            "config": {"workload": name, **{k: cfg[k] for k in cfg if k not in ("index", "kind")},
-                       "mu": args.mu, "variant": args.variant, "layout": layout,
-                       "append": (("fused into the eviction (vd_append_evict_decode)"
-                                   if isinstance(w, Decode) else
-                                   "fused into the eviction (vd_append_evict_block)")
-                                  if getattr(w, "fused", False) else "vd_append, then the eviction"),
-                       "l2": f"inputs larger than L2: cache {w.cache.k.numel() * 4 / 2**30:.2f} GiB "
-                             "of K+V, touched every step", "storage": "bf16"},
+            "roofline": stricter({
+                "bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                "frac": achieved / peak, "traffic": traffic, "kernel": kernel,
+                "algorithmic_bytes_per_launch": alg, "nominal_bytes_per_launch": nominal,
+                "bytes_breakdown": dict(w.breakdown), "moved_rows_per_launch": m["moved"],
+                "kernel_ms": kern_ms,
+                "peak_source": peak_src + ", of measured" if "measured" in peak_src else peak_src},
+                read_gbs),
+            "config": workload_config(name, cfg, mu_name, args.variant, layout,
+                                      getattr(w, "fused", False), isinstance(w, Decode)),
         }
+        if isinstance(w, RatioDecode):
+            res["config"]["budgets"] = (f"N_t = floor(L_t / 4), {w.budget[0]}..{w.budget[-1]} "
+                                        "over the timed window; 3 of 4 steps evict")
         return res
+
+    def brief(r):
+        """The parts of a measurement that go into the JSON line."""
+        out = {k: r[k] for k in ("value", "step_ms", "roofline", "e2e")}
+        out["mu"] = r["config"]["mu"]
+        return out
 
     def release(r):
         if r is not None:
             r.pop("w", None)
             torch.cuda.empty_cache()
 
+    summary = {}
+
+    def summarize(label, r):
+        rf = r["roofline"]
+        tr = rf.get("traffic")
+        summary[label] = [round(r["kern_ms"], 4), round(rf["frac"], 3), round(rf["frac_strict"], 3),
+                          round(tr / rf["algorithmic_bytes_per_launch"], 3) if tr else None,
+                          round(r["e2e"]["value"] / 1e9, 3)]
+
     primary = one(args.workload, args.steps, args.layout)
+    summarize(f"{args.workload} ({primary['config']['mu']} mean)", primary)
     base = None
     if rank == 0 and not args.no_cpu_baseline:
         base = cpu_baseline(primary["w"])
@@ -982,7 +1148,22 @@ def run_vd(args):
     secondary = None
     if args.secondary not in ("", "none") and args.secondary != args.workload:
         secondary = one(args.secondary, args.secondary_steps, args.layout)
+        summarize(f"{args.secondary} ({secondary['config']['mu']} mean)", secondary)
         release(secondary)
+    # the other configurations (and the paper's recomputed mean, Sec. 3.2
+    # Eq. vd, beside the running sum) measured the same way
+    configs = {}
+    if args.config_steps > 0 and args.layout == "ordered":
+        plan = [(n, None) for n in ("prefill_gqa8b", "ratio_budget")
+                if n not in (args.workload, args.secondary)]
+        other_mu = vd.VD_MU_RECOMPUTE if mu == vd.VD_MU_RUNNING else vd.VD_MU_RUNNING
+        plan += [(n, other_mu) for n in (args.workload, "prefill_gqa8b")]
+        for name, mm in plan:
+            r = one(name, args.config_steps, "ordered", mm)
+            label = f"{name} ({r['config']['mu']} mean)"
+            configs[label] = brief(r)
+            summarize(label, r)
+            release(r)
     # the same prefill step with a separate vd_append launch before the
     # eviction (the two-call form), for comparison with the fused step
     separate = None
@@ -1001,16 +1182,19 @@ def run_vd(args):
                    "kernel_us": r["kern_ms"] * 1e3, "e2e_event_us":
                    r["w"].head_tokens_per_step() * ws / r["e2e"]["value"] * 1e6,
                    "graph_event_us": graph_step_us(r["w"], args.latency_steps, device)}
+        summary["tiny_prefill us/event (eager, graph)"] = [round(latency["event_us"], 2),
+                                                           round(latency["graph_event_us"], 2)]
         release(r)
     # the hole-fill cache layout (a next row: same policy, fewest rows moved)
     holefill = {}
     if args.holefill_steps > 0 and args.layout == "ordered":
-        for name in (args.workload, args.secondary):
-            if name in ("", "none"):
+        for name in (args.workload, args.secondary, "prefill_gqa8b"):
+            if name in ("", "none") or name in holefill:
                 continue
             r = one(name, args.holefill_steps, "holefill")
+            holefill[name] = brief(r)
+            summarize(f"{name} hole-fill", r)
             release(r)
-            holefill[name] = {k: r[k] for k in ("value", "step_ms", "roofline", "e2e")}
     # scoring options on the primary (prefill) workload: the K-side rule (with
     # the running mean of K, as the primary's of V), attention weights, and the
     # per-unit dispersion sigma_V from a score-only pass, and as a by-product
@@ -1025,8 +1209,15 @@ def run_vd(args):
                                "roofline": r["roofline"]}
             if r["w"].sigma is not None:
                 extensions[key]["sigma_v_mean"] = float(r["w"].sigma.mean().item())
+            summarize(f"{args.workload} {key}", r)
             release(r)
-        extensions["dispersion"] = measure_dispersion(args, device, variant, peak, rank)
+        disp = measure_dispersion(args, device, variant, peak, rank)
+        stricter(disp["roofline"], read_gbs)
+        extensions["dispersion"] = disp
+        summary["sigma pass (running, recomputed mean)"] = [
+            round(disp["step_ms"], 4), round(disp["roofline"]["frac"], 3),
+            round(disp["recomputed_mean"]["step_ms"], 4),
+            round(disp["recomputed_mean"]["frac_of_peak"], 3)]
     if rank == 0:
         line = {
             "metric": METRIC, "value": primary["value"], "unit": UNIT, "n_gpus": ws,
@@ -1039,6 +1230,8 @@ def run_vd(args):
             "clocks": primary["m"]["clocks"],
             "gpu_launches": launches,
             "host_cpus": host_cpus,
+            "peaks_gbs": {"copy_measured": peak, "read_only_this_run": read_gbs,
+                          "nominal_hbm3e": NOMINAL_HBM_GBS},
         }
         if base is not None:
             line["cpu_baseline"] = base
@@ -1046,6 +1239,8 @@ def run_vd(args):
             line["secondary"] = {k: secondary[k] for k in ("workload", "value", "step_ms", "roofline",
                                                            "e2e", "config")}
             line["secondary"]["clocks"] = secondary["m"]["clocks"]
+        if configs:
+            line["configs"] = configs
         if separate is not None:
             line["separate_append"] = separate
         if latency is not None:
@@ -1054,6 +1249,10 @@ def run_vd(args):
             line["holefill_layout"] = holefill
         if extensions:
             line["extensions"] = extensions
+        # last, so that a reader of the line's tail sees every configuration
+        line["summary"] = {"columns": ["kernel_ms", "frac_of_copy_peak", "frac_strict",
+                                       "ncu_traffic_over_algorithmic", "e2e_G_head_tokens_per_s"],
+                           **summary}
         print(json.dumps(line), flush=True)
     if ws > 1:
         import torch.distributed as dist
@@ -1099,13 +1298,19 @@ def run_reference(args):
         total += time.perf_counter() - t0
     ms = total / args.steps * 1e3
     value = units * n / (ms / 1e3)
+    _, cfg0 = wl.config(args.workload)
+    if args.n_seq:
+        cfg0["n_seq"] = args.n_seq
     line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
             "impl": "reference",
-            "config": {"workload": name, "sample_units": units, "n": n, "N": N, "head_dim": d},
+            "config": workload_config(name, cfg0, args.mu, args.variant, args.layout,
+                                      not args.separate_append, cfg0["kind"] != "prefill"),
             "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
-                             "sample": f"{units} units of {name} per step at n={n} -> N={N}"},
+                             "cpu_model": cpu_model(),
+                             "sample": f"{units} of {wl.units_of(cfg0)} units of {name} per step "
+                                       f"at n={n} -> N={N} (fp64 C oracle, one thread per core)"},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
 
@@ -1126,6 +1331,8 @@ def main(argv=None):
                     help="steps of the key-side / weighted / dispersion measurements (0: skip)")
     ap.add_argument("--holefill-steps", type=int, default=50,
                     help="steps of the extra hole-fill-layout measurements (0: skip)")
+    ap.add_argument("--config-steps", type=int, default=50,
+                    help="steps of the other configurations and the other mean mode (0: skip)")
     ap.add_argument("--separate-append", action="store_true",
                     help="prefill steps append with vd_append, then evict (default: one "
                          "vd_append_evict_block call)")

@@ -157,3 +157,56 @@ def test_clock_sampler_without_samples_in_window():
     cs.mark(1.0, 1.01, 1.02)
     out = cs.stop()
     assert out["samples"] == 3 and out["samples_in_timed_region"] == 0
+
+
+def test_ratio_budget_accounting():
+    """Ratio budget: only the steps over their budget evict and count; rows
+    move from the evicted slot up to the step's own budget; the steps that
+    only append copy their new K and V rows in."""
+    U, d = 3, 8
+    w = object.__new__(bench.RatioDecode)
+    w.torch, w.U, w.N, w.d, w.mu = torch, U, 12, d, 1
+    w.record = [(11, 10), (11, 10), (11, 11), (12, 11)]    # n, N_t: the third step appends only
+    e = [torch.tensor(x, dtype=torch.int32) for x in ([0, 4, 10], [9, -1, 2], [-1, -1, -1],
+                                                       [11, 0, 5])]
+    assert w.moved_rows(e) == pytest.approx(((10 + 6 + 0) + (1 + 0 + 8) + 0 + (0 + 11 + 6)) / 4)
+    assert w.head_tokens_per_step() == pytest.approx(U * (11 + 11 + 12) / 4)
+    alg, nominal = w.bytes_per_launch(10.0)
+    v_read = U * d * 2 * (11 + 11 + 12) / 4
+    copy_in = U * d * 2 * 2 * 2 * 1 / 4
+    assert alg == pytest.approx(v_read + 10.0 * d * 8 + copy_in + U * d * 16)
+    assert nominal == pytest.approx(v_read + U * d * 8 * (10 + 10 + 11) / 4 + copy_in + U * d * 16)
+    assert set(w.breakdown) == {"scored_rows_read", "moved_rows_rw", "other"}
+
+
+def test_stricter_fractions():
+    r = bench.stricter({"achieved": 7300.0, "peak": 6789.0, "frac": 7300.0 / 6789.0}, 7100.0)
+    assert r["above_copy_peak"] is True
+    assert r["frac_of_read_peak"] == pytest.approx(7300 / 7100)
+    assert r["frac_strict"] == pytest.approx(7300 / bench.NOMINAL_HBM_GBS)
+    r = bench.stricter({"achieved": 5000.0, "peak": 6789.0, "frac": 5000 / 6789}, 8000.0)
+    assert r["above_copy_peak"] is False and r["frac_strict"] == pytest.approx(5000 / 8000)
+
+
+def test_cpu_model_names_arm_parts():
+    grace = "processor\t: 0\nBogoMIPS\t: 2000.00\nCPU implementer\t: 0x41\nCPU part\t: 0xd4f\n"
+    assert bench.cpu_model(grace).startswith("Arm Neoverse V2")
+    assert bench.cpu_model("model name\t: Some x86 CPU @ 2.0GHz\n") == "Some x86 CPU @ 2.0GHz"
+    assert bench.cpu_model("CPU implementer\t: 0x51\nCPU part\t: 0x001\n").startswith("part 0x001")
+
+
+def test_reference_arm_prints_the_workload_config(monkeypatch):
+    """Both arms describe the workload with the same config object."""
+    for k in ("WORLD_SIZE", "RANK", "LOCAL_RANK"):
+        monkeypatch.delenv(k, raising=False)
+    out = io.StringIO()
+    with contextlib.redirect_stdout(out):
+        bench.main(["--impl", "reference", "--workload", "tiny_prefill", "--steps", "1",
+                    "--warmup", "3"])
+    line = json.loads(out.getvalue().strip().splitlines()[-1])
+    from paper_2609_23314_gb300 import workloads as wl
+    _, cfg = wl.config("tiny_prefill")
+    want = bench.workload_config("tiny_prefill", cfg, "running", "l2", "ordered", True, False)
+    assert line["config"] == json.loads(json.dumps(want))
+    for k in ("n_seq", "n_layer", "n_kv_head", "head_dim", "T", "B", "N"):
+        assert line["config"][k] == cfg[k]
