@@ -11,8 +11,8 @@
 //             holds the same mean, kept as an fp32 part plus its remainder.
 //             Running-sum mode adds only the appended rows (spread over the
 //             cluster) to the caller's fp64 sum S.
-//   2. score  rows stream through a per-thread ring of asynchronous 16-byte
-//             copies (cp.async, 4 stages in flight); d/8 lanes per row, warp
+//   2. score  rows stream, last to first, through a per-thread ring of
+//             asynchronous 16-byte copies (cp.async, 4 stages); d/8 lanes per row, warp
 //             shuffle reduction of the squared deviation (L2, as
 //             ((v - hi) - lo)^2 against the two-part mean), of the norm
 //             (Norm), or of |w|^2 / (2 |v|^2) with w = v - (|v|/|mean|) mean
@@ -275,7 +275,9 @@ __device__ __forceinline__ float chunk_sq(const uint4& q, const unsigned long lo
 // ci holds row ci / (LPR / kBatch) of the batch: the lanes with
 // ci % (LPR / kBatch) == 0 call finish(j, s) for the batch's valid rows (j is
 // the row's index in [0, R)).  Same arithmetic per element as the general
-// path; only the order of the fp32 additions differs.
+// path; only the order of the fp32 additions differs.  Rows are visited from
+// the last to the first (see the score pass in evict_kernel).
+// R >= 1 (callers skip empty ranges).
 template <int VAR, int LPR, class Ring, int BATCH, class Finish>
 __device__ __forceinline__ void score_rows_fast(const uint16_t* __restrict__ rows, int R,
                                                 const float* mu, const float* mulo,
@@ -300,7 +302,8 @@ __device__ __forceinline__ void score_rows_fast(const uint16_t* __restrict__ row
   const int per_stage = kGroups * kItems;
   const int nst = (R + per_stage - 1) / per_stage;
   const uint32_t my = ring + (uint32_t)tid * 16u;
-  const uint16_t* p0 = rows + (size_t)g * kD + ci * 8;
+  // visit k of group g reads row R - 1 - (g + k * kGroups)
+  const uint16_t* p0 = rows + (size_t)(R - 1) * kD + ci * 8;
   auto slot = [&](int s, int u) {
     return my + (uint32_t)((s * kItems + u) * kThreads * 16);
   };
@@ -309,7 +312,8 @@ __device__ __forceinline__ void score_rows_fast(const uint16_t* __restrict__ row
 #pragma unroll
       for (int u = 0; u < kItems; ++u) {
         const int k = st * kItems + u;  // this group's k-th row: g + k * kGroups
-        if (g + k * kGroups < R) cp_async16(slot(st % kStages, u), p0 + (size_t)k * kGroups * kD);
+        const int i = g + k * kGroups;
+        if (i < R) cp_async16(slot(st % kStages, u), p0 - (size_t)i * kD);
       }
     }
     cp_async_commit();
@@ -347,7 +351,7 @@ __device__ __forceinline__ void score_rows_fast(const uint16_t* __restrict__ row
     for (int off = kSpread / 2; off >= 1; off >>= 1) part[0] += __shfl_xor_sync(kFull, part[0], off);
     if (ci % kSpread == 0) {
       const int j = g + (b * kBatch + ci / kSpread) * kGroups;
-      if (j < R) finish(j, sqrtf(part[0]));
+      if (j < R) finish(R - 1 - j, sqrtf(part[0]));
     }
   }
   cp_async_wait<0>();
@@ -382,7 +386,10 @@ __device__ __forceinline__ void merge_columns(float (&hi)[8], float (&lo)[8], in
 // acc (zeroed here) <- sum over items [0, count) of sign(item) * (the row at
 // row_ptr(item)), restricted to 16-byte column chunks [chunk0, chunk0 +
 // nchunks).
-template <class Ring, class RowPtr, class SignOf>
+// PACKED: TwoSum on packed fp32 pairs (half the instructions); the scalar
+// form gives bit-identical sums and is kept where the packed one would not
+// fit the kernel's register budget (the Dir block kernels).
+template <class Ring, bool PACKED = true, class RowPtr, class SignOf>
 __device__ __forceinline__ void sum_rows(int chunk0, int nchunks, int P, int count,
                                          RowPtr row_ptr, SignOf sign_of, Smem& S, uint32_t ring) {
   S.acc_hi[threadIdx.x] = 0.f;
@@ -390,20 +397,45 @@ __device__ __forceinline__ void sum_rows(int chunk0, int nchunks, int P, int cou
   __syncthreads();
   const int ci = (threadIdx.x & 31) & (P - 1);
   const bool active = ci < nchunks;
+  // the columns of this lane's chunk as packed pairs (2k, 2k + 1); each
+  // element enters with TwoSum (ff2_accumulate), a row of sign -1 with its
+  // sign bits flipped (exactly sign_of(item) * x)
   float hi[8], lo[8];
+  if constexpr (PACKED) {
+    unsigned long long hi2[4], lo2[4];
 #pragma unroll
-  for (int k = 0; k < 8; ++k) hi[k] = lo[k] = 0.f;
-  stream_rows<Ring>(chunk0, nchunks, P, count, row_ptr,
-              [&](int item, bool in, const uint4& q) {
-                if (in && active) {
-                  float x[8];
-                  unpack8(q, x);
-                  const float sg = sign_of(item);
+    for (int k = 0; k < 4; ++k) hi2[k] = lo2[k] = 0ull;
+    stream_rows<Ring>(chunk0, nchunks, P, count, row_ptr,
+                      [&](int item, bool in, const uint4& q) {
+                        if (in && active) {
+                          const uint32_t flip = sign_of(item) < 0.f ? 0x80008000u : 0u;
+                          const uint32_t w[4] = {q.x ^ flip, q.y ^ flip, q.z ^ flip, q.w ^ flip};
 #pragma unroll
-                  for (int k = 0; k < 8; ++k) ff_accumulate(hi[k], lo[k], sg * x[k]);
-                }
-              },
-              ring);
+                          for (int k = 0; k < 4; ++k)
+                            ff2_accumulate(hi2[k], lo2[k], bf16x2_to_f2(w[k]));
+                        }
+                      },
+                      ring);
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      f2_unpack(hi2[k], hi[2 * k], hi[2 * k + 1]);
+      f2_unpack(lo2[k], lo[2 * k], lo[2 * k + 1]);
+    }
+  } else {
+#pragma unroll
+    for (int k = 0; k < 8; ++k) hi[k] = lo[k] = 0.f;
+    stream_rows<Ring>(chunk0, nchunks, P, count, row_ptr,
+                      [&](int item, bool in, const uint4& q) {
+                        if (in && active) {
+                          float x[8];
+                          unpack8(q, x);
+                          const float sg = sign_of(item);
+#pragma unroll
+                          for (int k = 0; k < 8; ++k) ff_accumulate(hi[k], lo[k], sg * x[k]);
+                        }
+                      },
+                      ring);
+  }
   merge_columns(hi, lo, P, active, (chunk0 + ci) * 8, S.acc_hi, S.acc_lo);
 }
 
@@ -784,6 +816,8 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
   const int d = a.d, d8 = d >> 3;
   const int seq = u / a.units_per_seq;
   constexpr bool fused = FUSED;  // the new rows are still in the staging buffers
+  // packed-pair row sums everywhere but the Dir block kernels (register budget)
+  constexpr bool kPackedSum = !(VAR == 1 && !DECODE);
   const int len0 = a.len[seq];
   const int n = len0 + (fused ? a.B : 0);
   const int Nb = a.N_dev ? a.N_dev[seq] : a.N;
@@ -853,7 +887,7 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
     if (DECODE && a.evicted_out && rank == 0 && tid == 0) a.evicted_out[u] = -1;
     if (a.mu_running && a.B > 0 && tchunks > 0) {
       const uint16_t* nb = srange(first_new, a.B);  // the new rows lie on one side
-      sum_rows<Ring>(tchunk0, tchunks, tp, a.B, [&](int i) { return nb + (size_t)i * d; },
+      sum_rows<Ring, kPackedSum>(tchunk0, tchunks, tp, a.B, [&](int i) { return nb + (size_t)i * d; },
                [](int) { return 1.f; }, S, ring);
       if (tid < tchunks * 8) {
         const int c = tchunk0 * 8 + tid;
@@ -884,7 +918,7 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
     // the running sum is loaded before the row sum, whose latency hides it
     const double rs_own = run && tid < d ? a.running_sum[(size_t)u * d + tid] : 0.0;
     const uint16_t* pb = srange(p0, cnt);  // nullptr only where the range straddles
-    sum_rows<Ring>(0, d8, lpr, cnt,
+    sum_rows<Ring, kPackedSum>(0, d8, lpr, cnt,
                    [&](int i) -> const uint16_t* {
                      if constexpr (FUSED) return pb ? pb + (size_t)i * d : srow(p0 + i);
                      else return pb + (size_t)i * d;
@@ -930,6 +964,11 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
   if (score_split) cluster_arrive();
 
   // ---- 2. scores -------------------------------------------------------
+  // The rows are visited from the last to the first: the mean's row sum
+  // (recomputed mean) and the appended rows (running mean) were read in
+  // ascending order just before, so the first rows scored are the ones most
+  // recently brought into L2, and the compaction, which walks up from the
+  // first evicted slot, starts with the rows scored last.
   // sigma of the L2 scores (host-checked; compiled into the L2 kernels only)
   const bool disp = VAR == 0 && a.disp_out != nullptr;
   {
@@ -995,13 +1034,13 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
       const int c_end = min(r1, max(r0, first_stage));
       auto run = [&](auto lanes) {
         constexpr int LPR = decltype(lanes)::value;
-        if (c_end > r0)
-          score_rows_fast<VAR, LPR, Ring, kScoreBatch>(sb + (size_t)r0 * d, c_end - r0, S.mu, S.mulo,
-                                          finish_row, ring);
         if (r1 > c_end)
           score_rows_fast<VAR, LPR, Ring, kScoreBatch>(
               snu + (size_t)(c_end - first_stage) * d, r1 - c_end, S.mu, S.mulo,
               [&](int j, float s) { finish_row(j + (c_end - r0), s); }, ring);
+        if (c_end > r0)
+          score_rows_fast<VAR, LPR, Ring, kScoreBatch>(sb + (size_t)r0 * d, c_end - r0, S.mu,
+                                                       S.mulo, finish_row, ring);
       };
       fast = true;
       if (d == 128) run(std::integral_constant<int, 16>{});
@@ -1010,11 +1049,12 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
       else fast = false;
     }
     const uint16_t* rb = srange(r0, r1 - r0);  // nullptr only where the range straddles
+    const int nr = r1 - r0;  // rows visited last to first, as in score_rows_fast
     if (!fast) stream_rows<Ring>(
-        0, d8, lpr, r1 - r0,
+        0, d8, lpr, nr,
         [&](int i) -> const uint16_t* {
-          if constexpr (FUSED) return rb ? rb + (size_t)i * d : srow(r0 + i);
-          else return rb + (size_t)i * d;
+          if constexpr (FUSED) return rb ? rb + (size_t)(nr - 1 - i) * d : srow(r1 - 1 - i);
+          else return rb + (size_t)(nr - 1 - i) * d;
         },
         [&](int item, bool in, const uint4& q) {
           float x[8];
@@ -1063,7 +1103,7 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
             for (int off = 1; off < lpr; off <<= 1) acc += __shfl_xor_sync(kFull, acc, off);
             s = (nv > 0.f && !mu_zero) ? (0.5f * acc) / nv : 1.f;
           }
-          if (in && ci == 0) finish_row(item, s);
+          if (in && ci == 0) finish_row(nr - 1 - item, s);
         },
         ring);
     if constexpr (VAR == 0) {
@@ -1201,7 +1241,7 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
       const int c = tchunk0 * 8 + tid;
       base = VAR != 2 ? S.snew[c] : a.running_sum[(size_t)u * d + c] + 0.0;
     }
-    sum_rows<Ring>(tchunk0, tchunks, tp, B + (n - Nb),
+    sum_rows<Ring, kPackedSum>(tchunk0, tchunks, tp, B + (n - Nb),
              [&](int i) {
                const int r =
                    i < B ? first_new + i : (DECODE ? e_first : (int)perm[Nb + (i - B)]);
