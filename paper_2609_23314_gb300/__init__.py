@@ -114,20 +114,24 @@ def _stream(stream):
 
 
 def _ptr(t, dtype, shape, what, device):
+    """The tensor's device pointer after checking its type, device, layout
+    and shape (so that no wrong pointer reaches the library)."""
     if t is None:
         return None
-    torch = _torch()
-    if not isinstance(t, torch.Tensor):
-        raise TypeError(f"{what} must be a torch tensor")
-    if t.dtype != dtype:
-        raise TypeError(f"{what} must be {dtype}, got {t.dtype}")
-    if t.device != device:
-        raise ValueError(f"{what} must live on {device}, got {t.device}")
-    if not t.is_contiguous():
-        raise ValueError(f"{what} must be contiguous")
-    if tuple(t.shape) != tuple(shape):
+    try:
+        ok = (t.dtype == dtype and t.get_device() == (device.index if device.type == "cuda" else -1)
+              and t.is_contiguous() and t.shape == shape)
+    except AttributeError:
+        raise TypeError(f"{what} must be a torch tensor") from None
+    if not ok:
+        if t.dtype != dtype:
+            raise TypeError(f"{what} must be {dtype}, got {t.dtype}")
+        if t.device != device:
+            raise ValueError(f"{what} must live on {device}, got {t.device}")
+        if not t.is_contiguous():
+            raise ValueError(f"{what} must be contiguous")
         raise ValueError(f"{what} must have shape {tuple(shape)}, got {tuple(t.shape)}")
-    return ctypes.c_void_p(t.data_ptr())
+    return t.data_ptr()
 
 
 def _check(code: int, where: str):

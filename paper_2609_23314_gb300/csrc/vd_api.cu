@@ -14,11 +14,15 @@
 
 #include "vd.h"
 #include "vd_evict.cuh"
+#include "vd_small.cuh"
 
 namespace vd {
 const void* evict_kernel_l2(bool decode, bool holefill, bool fused);
 const void* evict_kernel_dir(bool decode, bool holefill, bool fused);
 const void* evict_kernel_norm(bool decode, bool holefill, bool fused);
+const void* small_kernel_l2(bool decode, bool fused);
+const void* small_kernel_dir(bool decode, bool fused);
+const void* small_kernel_norm(bool decode, bool fused);
 }  // namespace vd
 
 using vd::kThreads;
@@ -137,6 +141,14 @@ const void* evict_kernel(vd_variant var, bool decode, bool holefill, bool fused)
   }
 }
 
+const void* small_kernel(vd_variant var, bool decode, bool fused) {
+  switch (var) {
+    case VD_SCORE_L2: return vd::small_kernel_l2(decode, fused);
+    case VD_SCORE_DIR: return vd::small_kernel_dir(decode, fused);
+    default: return vd::small_kernel_norm(decode, fused);
+  }
+}
+
 vd_status device_state(DeviceState** out) {
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) {
@@ -171,6 +183,15 @@ vd_status device_state(DeviceState** out) {
                 cudaSuccess)
           return VD_ERR_CUDA;
       }
+    for (int var = 0; var < 3; ++var)
+      for (int kind = 0; kind < 4; ++kind) {
+        const void* kern = small_kernel((vd_variant)var, (kind & 1) != 0, (kind & 2) != 0);
+        if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 st.smem_optin) != cudaSuccess ||
+            cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) !=
+                cudaSuccess)
+          return VD_ERR_CUDA;
+      }
     st.ready = true;
   }
   *out = &st;
@@ -196,10 +217,10 @@ int lanes_per_row(int d) {
   return p;
 }
 
-bool cluster_fits(const void* kern, long long units, int c, size_t smem) {
+bool cluster_fits(const void* kern, long long groups, int c, size_t smem) {
   if (c == 1) return true;
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3((unsigned)(units * c));
+  cfg.gridDim = dim3((unsigned)(groups * c));
   cfg.blockDim = dim3(kThreads);
   cfg.dynamicSmemBytes = smem;
   cudaLaunchAttribute attr;
@@ -316,10 +337,58 @@ int cached_cluster(const void* kern, long long units, int d, int capacity, bool 
   return c;
 }
 
-vd_status launch(const void* kern, long long units, int c, size_t smem, const vd::EvictArgs& a,
+// The short-cache kernel (vd_small.cuh) takes a block or decode event when
+// the unit's K and V rows fit in shared memory with room to spare
+// (capacity * head_dim * 4 bytes <= kSmallRowBytes, capacity <= 1024), a
+// sequence's units fit in one cluster (<= 16), the launch is at most two
+// waves of one CTA per SM, and no scoring option, hole-fill layout or forced
+// cluster size (VD_CLUSTER_SIZE) is asked for.  VD_SMALL_PATH=0 turns it
+// off.  The choice depends on the shape only, so the fused and two-call
+// forms, block and decode, take the same kernel.
+constexpr size_t kSmallRowBytes = 64 * 1024;
+
+bool cluster_fits(const void* kern, long long groups, int c, size_t smem);
+
+bool use_small(const vd_cache* c, bool score_only, bool holefill, const float* weights,
+               const float* disp_out, int score_k, const DeviceState& st) {
+  if (score_only || holefill || weights || disp_out || score_k) return false;
+  const char* off = std::getenv("VD_SMALL_PATH");
+  if ((off && std::atoi(off) == 0) || std::getenv("VD_CLUSTER_SIZE")) return false;
+  const int ups = c->n_layer * c->n_kv_head;
+  const long long units = (long long)c->n_seq * ups;
+  if (ups > 16 || c->capacity > vd::kSmallMaxRows || units > 2LL * st.sms) return false;
+  if ((size_t)c->capacity * c->head_dim * 4 > kSmallRowBytes) return false;
+  return vd::small_layout(c->capacity, c->head_dim).total <= (size_t)st.smem_optin;
+}
+
+// groups clusters of c CTAs: the fused kernel's grid is units x c CTAs (a
+// cluster per unit), the short-cache kernel's n_seq x units_per_seq (a
+// cluster per sequence, a CTA per unit)
+// cluster_fits, remembered per launch shape (the occupancy query costs
+// several microseconds of host time, as much as a short-cache event takes on
+// the device); entries are marked with_select == 2 in the choice cache.
+bool cached_fits(const void* kern, long long groups, int c, size_t smem, DeviceState& st) {
+  {
+    std::lock_guard<std::mutex> lk(g_mu);
+    for (int i = 0; i < st.n_choice; ++i) {
+      const ClusterChoice& e = st.choice[i];
+      if (e.kern == kern && e.units == groups && e.with_select == 2 && e.want == c &&
+          e.smem == smem)
+        return e.c != 0;
+    }
+  }
+  const bool fits = c == 1 || cluster_fits(kern, groups, c, smem);
+  std::lock_guard<std::mutex> lk(g_mu);
+  st.choice[st.next_choice] = ClusterChoice{kern, groups, 0, 0, 2, c, fits ? c : 0, smem};
+  st.next_choice = (st.next_choice + 1) % kChoiceSlots;
+  if (st.n_choice < kChoiceSlots) ++st.n_choice;
+  return fits;
+}
+
+vd_status launch(const void* kern, long long groups, int c, size_t smem, const void* params,
                  cudaStream_t s) {
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3((unsigned)(units * c));
+  cfg.gridDim = dim3((unsigned)(groups * c));
   cfg.blockDim = dim3(kThreads);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = s;
@@ -330,7 +399,7 @@ vd_status launch(const void* kern, long long units, int c, size_t smem, const vd
   attr.val.clusterDim.z = 1;
   cfg.attrs = &attr;
   cfg.numAttrs = 1;
-  void* args[] = {const_cast<vd::EvictArgs*>(&a)};
+  void* args[] = {const_cast<void*>(params)};
   if (cudaLaunchKernelExC(&cfg, kern, args) != cudaSuccess) {
     cudaGetLastError();
     return VD_ERR_CUDA;
@@ -403,11 +472,22 @@ vd_status run(const vd_cache* c, int32_t N, const int32_t* N_dev, int32_t B, vd_
   a.disp_out = disp_out;
   a.k_new = static_cast<const uint16_t*>(k_new);
   a.v_new = static_cast<const uint16_t*>(v_new);
+  if (use_small(c, score_only, holefill, weights, disp_out, score_k, *st)) {
+    // one launch: the kernel also sets the sequences' lengths
+    // grid: n_seq clusters of units_per_seq CTAs, one CTA per unit
+    const void* sk = small_kernel(var, decode, fused);
+    const size_t ssmem = vd::small_layout(c->capacity, c->head_dim).total;
+    a.cluster = a.units_per_seq;
+    if (cached_fits(sk, c->n_seq, a.cluster, ssmem, *st)) {
+      const vd::SmallArgs sa{a, (int32_t)units};
+      return launch(sk, c->n_seq, a.cluster, ssmem, &sa, s);
+    }
+  }
   size_t smem = 0;
   a.cluster = cached_cluster(kern, units, c->head_dim, c->capacity, !small, holefill, *st, &smem);
   if (smem > (size_t)st->smem_optin) return VD_ERR_UNSUPPORTED;
 
-  r = launch(kern, units, a.cluster, smem, a, s);
+  r = launch(kern, units, a.cluster, smem, &a, s);
   if (r != VD_OK || score_only) return r;
   const int threads = 256;
   vd_len_clamp_kernel<<<(c->n_seq + threads - 1) / threads, threads, 0, s>>>(

@@ -107,7 +107,7 @@ __host__ __device__ constexpr int ring_bytes(bool with_select) {
 struct EvictArgs {
   uint16_t* k;            // bf16 [U][capacity][d]
   uint16_t* v;            // bf16 [U][capacity][d]
-  const int32_t* len;     // [n_seq]
+  int32_t* len;           // [n_seq] (written only by the short-cache kernel)
   const int32_t* N_dev;   // nullable [n_seq]
   double* running_sum;    // [U][d] (running mode)
   int32_t* kept_out;      // nullable [U][N]

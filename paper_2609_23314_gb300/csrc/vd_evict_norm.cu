@@ -1,6 +1,8 @@
-// vd_evict_norm.cu -- instantiates the fused eviction kernel for one scoring
-// rule (compiled separately so the translation units build in parallel).
+// vd_evict_norm.cu -- instantiates the fused eviction kernel and the short-cache
+// kernel for one scoring rule (compiled separately so the translation units
+// build in parallel).
 #include "vd_evict.cuh"
+#include "vd_small.cuh"
 
 namespace vd {
 const void* evict_kernel_norm(bool decode, bool holefill, bool fused) {
@@ -14,5 +16,14 @@ const void* evict_kernel_norm(bool decode, bool holefill, bool fused) {
        {reinterpret_cast<const void*>(&evict_kernel<2, true, true, false>),
         reinterpret_cast<const void*>(&evict_kernel<2, true, true, true>)}}};
   return k[decode][holefill][fused];
+}
+
+const void* small_kernel_norm(bool decode, bool fused) {
+  const void* k[2][2] = {
+      {reinterpret_cast<const void*>(&small_evict_kernel<2, false, false>),
+       reinterpret_cast<const void*>(&small_evict_kernel<2, false, true>)},
+      {reinterpret_cast<const void*>(&small_evict_kernel<2, true, false>),
+       reinterpret_cast<const void*>(&small_evict_kernel<2, true, true>)}};
+  return k[decode][fused];
 }
 }  // namespace vd

@@ -124,3 +124,26 @@ def test_scoring_options_rejected_before_launch(lib):
                                        None) == 1
     assert lib.vd_evict_decode_holefill(ref, 16, None, 0, 0, None, None, 0x40, None, None,
                                         None, None) == 1
+
+
+def test_binding_checks_every_tensor_argument():
+    """The binding passes a pointer only for a tensor of the expected dtype,
+    device, shape and layout; anything else raises before the library is
+    called."""
+    import torch
+    import paper_2609_23314_gb300 as vd
+    cuda0 = torch.device("cuda", 0)
+    cpu = torch.device("cpu")
+    t = torch.zeros(2, 3, dtype=torch.float32)
+    assert vd._ptr(None, torch.float32, (2, 3), "x", cpu) is None
+    assert vd._ptr(t, torch.float32, (2, 3), "x", cpu) == t.data_ptr()
+    with pytest.raises(TypeError):
+        vd._ptr(t, torch.int32, (2, 3), "x", cpu)
+    with pytest.raises(TypeError):
+        vd._ptr([1, 2], torch.float32, (2,), "x", cpu)
+    with pytest.raises(ValueError, match="live on"):
+        vd._ptr(t, torch.float32, (2, 3), "x", cuda0)
+    with pytest.raises(ValueError, match="contiguous"):
+        vd._ptr(t.t(), torch.float32, (3, 2), "x", cpu)
+    with pytest.raises(ValueError, match="shape"):
+        vd._ptr(t, torch.float32, (3, 2), "x", cpu)
