@@ -33,9 +33,17 @@
  *   word (read it with vd_get_device_status) and leaves the affected unit
  *   untouched, except VD_ERR_NONFINITE, which is recorded while the unit is
  *   still evicted with NaN scores ranked lowest.
- * - Precision: scores are computed in fp32 from bf16 inputs; the cache mean
- *   is accumulated with compensated fp32 sums (or kept as an fp64 running
- *   sum) so that it is correct to about 1e-7 relative.
+ * - Precision: scores are computed in fp32 from bf16 inputs against the
+ *   cache mean carried as an fp32 part plus its fp32 remainder; the mean is
+ *   accumulated with exact (TwoSum) fp32 sums, or from the fp64 running sum,
+ *   to about 1e-12 of the data's scale.  Every score's rounding error is
+ *   relative to the score itself (a few 1e-7 in practice).  Ranking: a NaN
+ *   score ranks below every number, +0 and -0 are equal.
+ * - Launches: one eviction kernel per call, plus a one-thread-per-sequence
+ *   length update.  A short cache (capacity <= 1024, 4 * capacity * head_dim
+ *   <= 64 KB, at most 16 units per sequence, at most two units per SM) takes
+ *   a kernel that keeps the unit in shared memory and updates the lengths
+ *   itself: one launch in all.  Results follow the same rules either way.
  */
 #ifndef VD_H
 #define VD_H

@@ -23,12 +23,20 @@ def pytest_terminal_summary(terminalreporter):
     """The worst score error each GPU test saw against the oracle, per rule:
     relative (over scores above 1e-6) and as a fraction of the tolerance."""
     try:
-        from vd_gpu import WORST
+        from vd_gpu import TRAJECTORIES, WORST
     except Exception:
         return
+    tr = terminalreporter
+    if TRAJECTORIES:
+        tr.section("free-running trajectories, CUDA path vs the oracle's own loop")
+        for name, t in sorted(TRAJECTORIES.items()):
+            fd = t["first_divergence"]
+            tr.write_line(f"{name:<16} {t['units']} units, {t['events']} evicting events: "
+                          f"{t['identical_events']} identical, first divergence "
+                          f"{'none' if fd is None else f'event {fd[0]} (unit {fd[1]})'}, "
+                          f"final caches share {100 * t['final_overlap']:.1f} % of their tokens")
     if not WORST:
         return
-    tr = terminalreporter
     tr.section("worst score error vs the fp64 oracle (tolerance 1e-5 relative)")
     for (test, rule), (rel, frac, count) in sorted(WORST.items()):
         tr.write_line(f"{test:<60} {rule:<8} rel {rel:.2e}  of tol {frac:.3f}  ({count} scores)")

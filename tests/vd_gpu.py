@@ -37,6 +37,8 @@ DIR_RADIAL_FLOOR = 0.5 * (32 * 2.0 ** -24) ** 2
 
 # (test, rule) -> [worst |ds| / s over scores > 1e-6, worst |ds| / tolerance, count]
 WORST: dict = {}
+# workload -> summary of a free-running trajectory (test_gpu_trajectory.py)
+TRAJECTORIES: dict = {}
 
 
 def record_error(var, s_gpu, s_ora, tag: str = "", tol=None):
