@@ -70,7 +70,8 @@ typedef enum {
                              C <= head_dim / 4): at head_dim >= 64 every
                              capacity up to 65536 fits */
   VD_ERR_NONFINITE = 4,   /* device: a score was NaN or infinite */
-  VD_ERR_TIMEOUT = 5,     /* reserved: no kernel in this library waits on a flag */
+  VD_ERR_TIMEOUT = 5,     /* device: a bounded wait for a bulk copy gave up (score-only
+                             kernels); that call's outputs are unspecified */
   VD_ERR_CUDA = 6,        /* a CUDA runtime call failed (launch error, ...) */
   VD_ERR_DEVICE_LEN = 7,  /* device: len[s] out of [0, capacity], or len + B > capacity
                              on append, or B > len in running-sum mode */

@@ -23,6 +23,9 @@ const void* evict_kernel_norm(bool decode, bool holefill, bool fused);
 const void* small_kernel_l2(bool decode, bool fused);
 const void* small_kernel_dir(bool decode, bool fused);
 const void* small_kernel_norm(bool decode, bool fused);
+const void* score_kernel_l2();
+const void* score_kernel_dir();
+const void* score_kernel_norm();
 }  // namespace vd
 
 using vd::kThreads;
@@ -91,7 +94,7 @@ __global__ void __launch_bounds__(kThreads) vd_rsum_init_kernel(const uint16_t* 
                                                                 unsigned* status) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   vd::Smem& S = *reinterpret_cast<vd::Smem*>(smem_raw);
-  const uint32_t ring = vd::smem_addr(smem_raw + vd::smem_layout(cap, 1, false).ring);
+  const uint32_t ring = vd::smem_addr(smem_raw + vd::smem_layout(cap, 1, vd::kKindDecode).ring);
   const int u = blockIdx.x;
   const int n = len[u / units_per_seq];
   if (n < 0 || n > cap) {
@@ -115,7 +118,7 @@ namespace {
 struct ClusterChoice {
   const void* kern;
   long long units;
-  int d, capacity, with_select, want, c;
+  int d, capacity, kind, want, c;  // kind: vd::kKind*, or kFitsKind (cached_fits)
   size_t smem;
 };
 constexpr int kChoiceSlots = 32;
@@ -138,6 +141,14 @@ const void* evict_kernel(vd_variant var, bool decode, bool holefill, bool fused)
     case VD_SCORE_L2: return vd::evict_kernel_l2(decode, holefill, fused);
     case VD_SCORE_DIR: return vd::evict_kernel_dir(decode, holefill, fused);
     default: return vd::evict_kernel_norm(decode, holefill, fused);
+  }
+}
+
+const void* score_kernel(vd_variant var) {
+  switch (var) {
+    case VD_SCORE_L2: return vd::score_kernel_l2();
+    case VD_SCORE_DIR: return vd::score_kernel_dir();
+    default: return vd::score_kernel_norm();
   }
 }
 
@@ -184,8 +195,10 @@ vd_status device_state(DeviceState** out) {
           return VD_ERR_CUDA;
       }
     for (int var = 0; var < 3; ++var)
-      for (int kind = 0; kind < 4; ++kind) {
-        const void* kern = small_kernel((vd_variant)var, (kind & 1) != 0, (kind & 2) != 0);
+      for (int kind = 0; kind < 5; ++kind) {
+        const void* kern = kind == 4 ? score_kernel((vd_variant)var)
+                                     : small_kernel((vd_variant)var, (kind & 1) != 0,
+                                                    (kind & 2) != 0);
         if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  st.smem_optin) != cudaSuccess ||
             cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) !=
@@ -254,7 +267,11 @@ bool cluster_allowed(int c, int d) {
 // 0.4 of a wave (one short wave beats a long tail and more cluster barriers:
 // prefill_wide C=1, 0.74 waves, 0.211-0.216 ms vs C=2, 1.47 waves,
 // 0.216-0.221; prefill_gqa8b C=1, 0.47 waves, 0.064 ms vs C=2, 0.95 waves,
-// 0.069).  With none such (few units), the largest allowed C that
+// 0.069).  Score-only launches on the bulk-copy ring: the smallest C with at
+// least half a wave (fewer, longer contiguous slices: the prefill_wide sigma
+// pass at C=1, 0.74 waves, 0.115 ms vs C=2 0.131, C=4 0.139; 2 ring stages at
+// 3 CTAs per SM; 3 stages 0.141 ms, 4 stages 0.149).  With none such (few
+// units), the largest allowed C that
 // leaves every CTA at least kMinRowsPerCta rows of the capacity, else the
 // smallest allowed C: below that, the cluster barriers cost more than the
 // split saves.  (Measured on GB300: prefill_wide ordered C=8 (4.4 waves)
@@ -266,13 +283,14 @@ bool cluster_allowed(int c, int d) {
 // (VD_CLUSTER_SIZE: 1, 2, 4, 8 or 16) overrides the choice, for tuning.
 constexpr int kMinRowsPerCta = 128;
 
-int choose_cluster(const void* kern, long long units, int d, int capacity, bool with_select,
+int choose_cluster(const void* kern, long long units, int d, int capacity, int kind,
                    bool holefill, int want, const DeviceState& st, size_t* smem_out) {
+  const bool with_select = kind == vd::kKindBlock;
   int chosen = 0, fallback = 0, roomy = 0, smallest = 0, narrow = 0;
   for (int c = 1; c <= 16; c *= 2) {
     if (want >= 1 && c != want) continue;
     if ((d / 8 * 2) % c) continue;
-    const size_t smem = vd::smem_layout(capacity, c, with_select).total;
+    const size_t smem = vd::smem_layout(capacity, c, kind).total;
     if (smem > (size_t)st.smem_optin) continue;
     int occ = 0;
     if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, kern, kThreads, smem) != cudaSuccess) {
@@ -295,6 +313,8 @@ int choose_cluster(const void* kern, long long units, int d, int capacity, bool 
       ok = true;
     else if (with_select && holefill)
       ok = waves >= 0.4;
+    else if (kind == vd::kKindScoreBulk)
+      ok = waves >= 0.5;
     else if (with_select)
       ok = full_wave || waves >= 4.0;
     else
@@ -307,31 +327,30 @@ int choose_cluster(const void* kern, long long units, int d, int capacity, bool 
   }
   if (chosen == 0)
     chosen = fallback ? fallback : roomy ? roomy : smallest ? smallest : narrow ? narrow : 1;
-  *smem_out = vd::smem_layout(capacity, chosen, with_select).total;
+  *smem_out = vd::smem_layout(capacity, chosen, kind).total;
   return chosen;
 }
 
 // choose_cluster, remembered per launch shape.
-int cached_cluster(const void* kern, long long units, int d, int capacity, bool with_select,
+int cached_cluster(const void* kern, long long units, int d, int capacity, int kind,
                    bool holefill, DeviceState& st, size_t* smem_out) {
   const char* env = std::getenv("VD_CLUSTER_SIZE");
   const int want = env ? std::atoi(env) : 0;
-  const int ws = with_select ? 1 : 0;
   {
     std::lock_guard<std::mutex> lk(g_mu);
     for (int i = 0; i < st.n_choice; ++i) {
       const ClusterChoice& e = st.choice[i];
       if (e.kern == kern && e.units == units && e.d == d && e.capacity == capacity &&
-          e.with_select == ws && e.want == want) {
+          e.kind == kind && e.want == want) {
         *smem_out = e.smem;
         return e.c;
       }
     }
   }
-  const int c = choose_cluster(kern, units, d, capacity, with_select, holefill, want, st,
+  const int c = choose_cluster(kern, units, d, capacity, kind, holefill, want, st,
                                smem_out);
   std::lock_guard<std::mutex> lk(g_mu);
-  st.choice[st.next_choice] = ClusterChoice{kern, units, d, capacity, ws, want, c, *smem_out};
+  st.choice[st.next_choice] = ClusterChoice{kern, units, d, capacity, kind, want, c, *smem_out};
   st.next_choice = (st.next_choice + 1) % kChoiceSlots;
   if (st.n_choice < kChoiceSlots) ++st.n_choice;
   return c;
@@ -366,20 +385,21 @@ bool use_small(const vd_cache* c, bool score_only, bool holefill, const float* w
 // cluster per sequence, a CTA per unit)
 // cluster_fits, remembered per launch shape (the occupancy query costs
 // several microseconds of host time, as much as a short-cache event takes on
-// the device); entries are marked with_select == 2 in the choice cache.
+// the device); entries are marked kind == kFitsKind in the choice cache.
+constexpr int kFitsKind = 3;
 bool cached_fits(const void* kern, long long groups, int c, size_t smem, DeviceState& st) {
   {
     std::lock_guard<std::mutex> lk(g_mu);
     for (int i = 0; i < st.n_choice; ++i) {
       const ClusterChoice& e = st.choice[i];
-      if (e.kern == kern && e.units == groups && e.with_select == 2 && e.want == c &&
+      if (e.kern == kern && e.units == groups && e.kind == kFitsKind && e.want == c &&
           e.smem == smem)
         return e.c != 0;
     }
   }
   const bool fits = c == 1 || cluster_fits(kern, groups, c, smem);
   std::lock_guard<std::mutex> lk(g_mu);
-  st.choice[st.next_choice] = ClusterChoice{kern, groups, 0, 0, 2, c, fits ? c : 0, smem};
+  st.choice[st.next_choice] = ClusterChoice{kern, groups, 0, 0, kFitsKind, c, fits ? c : 0, smem};
   st.next_choice = (st.next_choice + 1) % kChoiceSlots;
   if (st.n_choice < kChoiceSlots) ++st.n_choice;
   return fits;
@@ -438,12 +458,15 @@ vd_status run(const vd_cache* c, int32_t N, const int32_t* N_dev, int32_t B, vd_
   r = device_state(&st);
   if (r != VD_OK) return r;
 
-  // score-only uses the decode instantiation: it needs no per-token buffers
-  const bool small = decode || score_only;
-  if (!small && c->capacity > 65536) return VD_ERR_UNSUPPORTED;  // 16-bit slot lists
-  if (vd::smem_layout(c->capacity, 16, !small).total > (size_t)st->smem_optin)
+  // score-only launches have their own instantiation (no per-token buffers)
+  const int kind = score_only ? (vd::score_bulk((int)var, c->head_dim) ? vd::kKindScoreBulk
+                                                                       : vd::kKindScore)
+                 : decode     ? vd::kKindDecode
+                              : vd::kKindBlock;
+  if (kind == vd::kKindBlock && c->capacity > 65536) return VD_ERR_UNSUPPORTED;  // 16-bit lists
+  if (vd::smem_layout(c->capacity, 16, kind).total > (size_t)st->smem_optin)
     return VD_ERR_UNSUPPORTED;
-  const void* kern = evict_kernel(var, small, holefill, fused);
+  const void* kern = score_only ? score_kernel(var) : evict_kernel(var, decode, holefill, fused);
   const long long units = (long long)c->n_seq * c->n_layer * c->n_kv_head;
 
   vd::EvictArgs a;
@@ -484,7 +507,7 @@ vd_status run(const vd_cache* c, int32_t N, const int32_t* N_dev, int32_t B, vd_
     }
   }
   size_t smem = 0;
-  a.cluster = cached_cluster(kern, units, c->head_dim, c->capacity, !small, holefill, *st, &smem);
+  a.cluster = cached_cluster(kern, units, c->head_dim, c->capacity, kind, holefill, *st, &smem);
   if (smem > (size_t)st->smem_optin) return VD_ERR_UNSUPPORTED;
 
   r = launch(kern, units, a.cluster, smem, &a, s);
@@ -629,7 +652,7 @@ vd_status vd_running_sum_init_ex(const vd_cache* c, int32_t of_keys, double* run
   r = device_state(&st);
   if (r != VD_OK) return r;
   const long long units = (long long)c->n_seq * c->n_layer * c->n_kv_head;
-  const size_t smem = vd::smem_layout(c->capacity, 1, false).total;
+  const size_t smem = vd::smem_layout(c->capacity, 1, vd::kKindDecode).total;
   vd_rsum_init_kernel<<<(unsigned)units, kThreads, smem, reinterpret_cast<cudaStream_t>(stream)>>>(
       static_cast<const uint16_t*>(of_keys ? c->k : c->v), c->len, running_sum,
       c->n_layer * c->n_kv_head,

@@ -16,6 +16,7 @@ constexpr unsigned kFull = 0xffffffffu;
 
 // Device status codes (the values of vd_status in include/vd.h).
 constexpr unsigned kStNonfinite = 4;
+constexpr unsigned kStTimeout = 5;
 constexpr unsigned kStDeviceLen = 7;
 constexpr unsigned kStDeviceBudget = 8;
 constexpr unsigned kStInternal = 10;
@@ -140,6 +141,60 @@ __device__ __forceinline__ void st16(void* p, const uint4& v) {
   asm volatile("st.global.v4.u32 [%0], {%1,%2,%3,%4};" ::"l"(p), "r"(v.x), "r"(v.y), "r"(v.z),
                "r"(v.w)
                : "memory");
+}
+
+// ---------------------------------------------------------------------------
+// Bulk copies: one thread moves a contiguous block of global memory into this
+// CTA's own shared memory (cp.async.bulk, no multicast; both addresses and the
+// size multiples of 16 bytes), and the copy's completion is counted on an
+// mbarrier in shared memory (expect_tx bytes, complete_tx by the copy).
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ void mbar_init(uint32_t bar, unsigned count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+
+// Makes barrier initialisations visible to the copy engine (and the cluster).
+__device__ __forceinline__ void fence_mbar_init() {
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+
+// Orders this thread's earlier shared-memory accesses before later bulk-copy
+// writes into the same memory.
+__device__ __forceinline__ void fence_proxy_async_smem() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
+               : "memory");
+}
+
+__device__ __forceinline__ void bulk_g2s(uint32_t dst, const void* src, uint32_t bytes,
+                                         uint32_t bar) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+      ::"r"(dst), "l"(src), "r"(bytes), "r"(bar)
+      : "memory");
+}
+
+// Waits until the barrier's phase with the given parity has completed, for
+// at most `limit` polls.  Returns false (and records kStTimeout) if it gave
+// up: the caller then goes on with whatever the buffer holds, so that the
+// kernel still ends and every barrier of the CTA or cluster is still reached.
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, unsigned* status,
+                                          unsigned limit = 1u << 22) {
+  for (unsigned i = 0; i < limit; ++i) {
+    uint32_t done;
+    asm volatile(
+        "{ .reg .pred p; mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2; "
+        "selp.u32 %0, 1, 0, p; }"
+        : "=r"(done)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    if (done) return true;
+  }
+  record_status(status, kStTimeout);
+  return false;
 }
 
 // ---------------------------------------------------------------------------

@@ -89,6 +89,23 @@ namespace vd {
 #ifndef VD_DECODE_MIN_CTAS
 #define VD_DECODE_MIN_CTAS 4
 #endif
+// Score-only launches (vd_score, vd_score_ex) have their own instantiation:
+// no select, slot lists or compaction, so a deeper ring fits at a lower
+// occupancy.
+#ifndef VD_SCORE_RING_STAGES
+#define VD_SCORE_RING_STAGES 8
+#endif
+#ifndef VD_SCORE_RING_ITEMS
+#define VD_SCORE_RING_ITEMS 2
+#endif
+#ifndef VD_SCORE_MIN_CTAS
+#define VD_SCORE_MIN_CTAS 3
+#endif
+// Score-only launches at head dims 64, 128, 256 (L2, Norm) stream through a
+// ring of bulk copies instead: VD_SCORE_BULK_STAGES stages of 32 KB.
+#ifndef VD_SCORE_BULK_STAGES
+#define VD_SCORE_BULK_STAGES 2
+#endif
 template <int STAGES, int ITEMS>
 struct RingShape {
   static constexpr int kStages = STAGES;
@@ -97,11 +114,25 @@ struct RingShape {
 };
 using BlockRing = RingShape<VD_RING_STAGES, VD_RING_ITEMS>;
 using DecodeRing = RingShape<VD_DECODE_RING_STAGES, VD_DECODE_RING_ITEMS>;
+using ScoreRing = RingShape<VD_SCORE_RING_STAGES, VD_SCORE_RING_ITEMS>;
 
-// Ring bytes of a launch: block eviction (with the select) or decode /
-// score-only.
-__host__ __device__ constexpr int ring_bytes(bool with_select) {
-  return with_select ? BlockRing::kBytes : DecodeRing::kBytes;
+// Launch kinds, which size the shared memory: decode eviction, block
+// eviction (the select's keys and the slot list too), score-only.
+constexpr int kKindDecode = 0, kKindBlock = 1, kKindScore = 2, kKindScoreBulk = 3;
+constexpr int kBulkStages = VD_SCORE_BULK_STAGES;
+constexpr int kBulkStageBytes = 32768;
+
+__host__ __device__ constexpr int ring_bytes(int kind) {
+  return kind == kKindBlock        ? BlockRing::kBytes
+         : kind == kKindScore      ? ScoreRing::kBytes
+         : kind == kKindScoreBulk  ? kBulkStages * kBulkStageBytes
+                                   : DecodeRing::kBytes;
+}
+
+// Whether a score-only launch takes the bulk ring: the batched L2 / Norm
+// score pass, whose stage of 32 KB is exactly one batch of rows per lane group.
+__host__ __device__ constexpr bool score_bulk(int var, int d) {
+  return var != 1 && (d == 64 || d == 128 || d == 256);
 }
 
 struct EvictArgs {
@@ -121,7 +152,7 @@ struct EvictArgs {
   int32_t N;              // scalar budget, kept_out stride, N_dev bound
   int32_t B;              // rows appended since the previous eviction
   int32_t mu_running;     // 1: mean from running_sum + appended rows
-  int32_t score_only;     // 1: vd_score / vd_score_ex (no eviction)
+  int32_t score_only;     // 1: vd_score / vd_score_ex (the kernels take it from SCORE)
   int32_t cluster;        // C, CTAs per unit
   int32_t* pos;            // hole-fill layout: token positions [U][capacity]
   const int32_t* pos_new;  // hole-fill layout: position of row len - B, [n_seq]
@@ -162,6 +193,7 @@ struct Smem {
   float inv_mnorm;     // Dir: 1 / |mean|
   float disp[4];       // dispersion partials: sum s (hi, lo), sum s^2 (hi, lo)
   float dsc[4 * kWarps];  // dispersion: per-warp partials (block-private)
+  unsigned long long bar[4];  // bulk ring: one mbarrier per stage (score-only)
 };
 
 __host__ __device__ constexpr size_t align16(size_t x) { return (x + 15) & ~(size_t)15; }
@@ -182,10 +214,11 @@ struct SmemLayout {
   size_t ring, keys, perm, total;
 };
 
-__host__ __device__ inline SmemLayout smem_layout(int capacity, int cluster, bool with_select) {
+__host__ __device__ inline SmemLayout smem_layout(int capacity, int cluster, int kind) {
+  const bool with_select = kind == kKindBlock;
   SmemLayout l;
   l.ring = (sizeof(Smem) + 127) & ~(size_t)127;
-  l.keys = l.ring + (size_t)ring_bytes(with_select);
+  l.keys = l.ring + (size_t)ring_bytes(kind);
   const size_t rows = with_select ? (size_t)((capacity + cluster - 1) / cluster) : 0;
   l.perm = l.keys + align16(rows * 4);
   l.total = l.perm + (with_select ? align16((size_t)capacity * 2) : 0);
@@ -437,6 +470,156 @@ __device__ __forceinline__ void sum_rows(int chunk0, int nchunks, int P, int cou
                       ring);
   }
   merge_columns(hi, lo, P, active, (chunk0 + ci) * 8, S.acc_hi, S.acc_lo);
+}
+
+static_assert(kBulkStages >= 2 && kBulkStages <= 4, "bulk ring: 2 to 4 stages (Smem::bar)");
+
+// A ring of bulk copies over this CTA's ring region: kBulkStages slots of
+// kBulkStageBytes, slot s completing on mbarrier Smem::bar[s].  gst counts
+// the stages started by every stream of the launch so far (the same value in
+// every thread): stage g uses slot g % S and waits for parity (g / S) & 1.
+struct BulkRing {
+  uint32_t ring, bar0;
+  int gst;
+};
+
+__device__ __forceinline__ BulkRing bulk_ring_init(uint32_t ring, Smem& S) {
+  const uint32_t bar0 = smem_addr(&S.bar[0]);
+  if (threadIdx.x == 0) {
+    for (int sl = 0; sl < kBulkStages; ++sl) mbar_init(bar0 + 8u * (uint32_t)sl, 1);
+    fence_mbar_init();
+  }
+  __syncthreads();
+  return {ring, bar0, 0};
+}
+
+// Streams nst stages of the rows at `base` (row_bytes each); stage_rows(i,
+// first, count) names stage i's rows [first, first + count).  Thread 0 issues
+// each stage as one bulk copy; every thread waits for it, consume(first,
+// count, stage address) reads it, and a block barrier frees the slot before
+// thread 0 refills it.
+template <class StageRows, class Consume>
+__device__ __forceinline__ void bulk_stream(BulkRing& br, const uint16_t* base, int nst,
+                                            int row_bytes, StageRows stage_rows, Consume consume,
+                                            unsigned* status) {
+  auto issue = [&](int i) {
+    int first, count;
+    stage_rows(i, first, count);
+    const uint32_t sl = (uint32_t)((br.gst + i) % kBulkStages);
+    const uint32_t bar = br.bar0 + 8u * sl;
+    const uint32_t bytes = (uint32_t)(count * row_bytes);
+    fence_proxy_async_smem();  // the slot's previous contents were read by generic loads
+    mbar_expect_tx(bar, bytes);
+    bulk_g2s(br.ring + sl * (uint32_t)kBulkStageBytes,
+             reinterpret_cast<const char*>(base) + (size_t)first * row_bytes, bytes, bar);
+  };
+  if (threadIdx.x == 0)
+    for (int i = 0; i < nst && i < kBulkStages; ++i) issue(i);
+  for (int i = 0; i < nst; ++i) {
+    const int g = br.gst + i;
+    const uint32_t sl = (uint32_t)(g % kBulkStages);
+    mbar_wait(br.bar0 + 8u * sl, (uint32_t)(g / kBulkStages) & 1u, status);
+    int first, count;
+    stage_rows(i, first, count);
+    consume(first, count, br.ring + sl * (uint32_t)kBulkStageBytes);
+    __syncthreads();  // every thread is done with the slot
+    if (threadIdx.x == 0 && i + kBulkStages < nst) issue(i + kBulkStages);
+  }
+  br.gst += nst;
+}
+
+// sum_rows over the contiguous rows [0, count) at `rows` (all d columns, P =
+// d / 8 lanes per row), streamed through the bulk ring in ascending order.
+// Lane group g takes rows g, g + 256/P, ... (a stage holds a whole number of
+// such strides), as sum_rows does, so the sums are bit-identical to it.
+__device__ __forceinline__ void sum_rows_bulk(BulkRing& br, const uint16_t* rows, int count,
+                                              int d, int P, Smem& S, unsigned* status) {
+  S.acc_hi[threadIdx.x] = 0.f;
+  S.acc_lo[threadIdx.x] = 0.f;
+  __syncthreads();
+  const int row_bytes = d * 2, srows = kBulkStageBytes / row_bytes;
+  const int ci = (threadIdx.x & 31) & (P - 1), g = threadIdx.x / P, ng = kThreads / P;
+  const bool active = ci < (d >> 3);
+  unsigned long long hi2[4], lo2[4];
+#pragma unroll
+  for (int k = 0; k < 4; ++k) hi2[k] = lo2[k] = 0ull;
+  bulk_stream(
+      br, rows, (count + srows - 1) / srows, row_bytes,
+      [&](int i, int& first, int& cnt) {
+        first = i * srows;
+        cnt = min(srows, count - first);
+      },
+      [&](int, int cnt, uint32_t st) {
+        if (!active) return;
+        for (int r = g; r < cnt; r += ng) {
+          const uint4 q = ld_shared16(st + (uint32_t)(r * row_bytes + ci * 16));
+          const uint32_t w[4] = {q.x, q.y, q.z, q.w};
+#pragma unroll
+          for (int k = 0; k < 4; ++k) ff2_accumulate(hi2[k], lo2[k], bf16x2_to_f2(w[k]));
+        }
+      },
+      status);
+  float hi[8], lo[8];
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    f2_unpack(hi2[k], hi[2 * k], hi[2 * k + 1]);
+    f2_unpack(lo2[k], lo[2 * k], lo[2 * k + 1]);
+  }
+  merge_columns(hi, lo, P, active, ci * 8, S.acc_hi, S.acc_lo);
+}
+
+// score_rows_fast through the bulk ring: a stage is one batch of 8 rows per
+// lane group (32 KB at d = 64, 128, 256), taken from the last rows to the
+// first; per row the same arithmetic as score_rows_fast.
+template <int VAR, int LPR, class Finish>
+__device__ __forceinline__ void score_rows_bulk(BulkRing& br, const uint16_t* rows, int R,
+                                                const float* mu, const float* mulo,
+                                                Finish finish, unsigned* status) {
+  constexpr int kBatch = 8, kGroups = kThreads / LPR, kD = LPR * 8, kSpread = LPR / kBatch;
+  constexpr int kRowBytes = kD * 2, kSRows = kBulkStageBytes / kRowBytes;
+  static_assert(kSRows == kGroups * kBatch, "one batch per lane group per stage");
+  const int tid = threadIdx.x, lane = tid & 31, ci = lane & (LPR - 1), g = tid / LPR;
+  unsigned long long m2[4];
+#pragma unroll
+  for (int k = 0; k < 4; ++k)
+    m2[k] = VAR == 0 ? f2_pack(mu[ci * 8 + 2 * k], mu[ci * 8 + 2 * k + 1]) : 0ull;
+  const uint32_t lo_addr = smem_addr(mulo) + (uint32_t)ci * 8u;
+  bulk_stream(
+      br, rows, (R + kSRows - 1) / kSRows, kRowBytes,
+      [&](int i, int& first, int& cnt) {
+        const int end = R - i * kSRows;
+        first = max(0, end - kSRows);
+        cnt = end - first;
+      },
+      [&](int first, int cnt, uint32_t st) {
+        float part[kBatch];
+#pragma unroll
+        for (int k = 0; k < kBatch; ++k) {
+          const int r = g + k * kGroups;
+          uint4 q = make_uint4(0u, 0u, 0u, 0u);
+          if (r < cnt) q = ld_shared16(st + (uint32_t)(r * kRowBytes + ci * 16));
+          part[k] = chunk_sq<VAR, LPR>(q, m2, lo_addr);
+        }
+#pragma unroll
+        for (int j = 0; j < 3; ++j) {
+          const int h = kBatch >> (j + 1), off = LPR >> (j + 1);
+          const bool upper = (ci & off) != 0;
+#pragma unroll
+          for (int k = 0; k < h; ++k) {
+            const float send = upper ? part[k] : part[k + h];
+            const float keep = upper ? part[k + h] : part[k];
+            part[k] = keep + __shfl_xor_sync(kFull, send, off);
+          }
+        }
+#pragma unroll
+        for (int off = kSpread / 2; off >= 1; off >>= 1)
+          part[0] += __shfl_xor_sync(kFull, part[0], off);
+        if (ci % kSpread == 0) {
+          const int r = g + (ci / kSpread) * kGroups;
+          if (r < cnt) finish(first + r, sqrtf(part[0]));
+        }
+      },
+      status);
 }
 
 // Order-preserving key of a score (scores are never negative): a positive
@@ -795,17 +978,27 @@ __device__ __forceinline__ void move_rows(uint16_t* kb, uint16_t* vb, int d, int
 // the radix select.  HF: hole-fill layout (compiled separately, so the ordered
 // layout carries none of its code).  FUSED: the new rows are read from the
 // caller's staging buffers (vd_append_evict_*); the other kernels carry none
-// of that code.
-template <int VAR, bool DECODE, bool HF, bool FUSED>
-__global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLOCK_MIN_CTAS)
+// of that code.  SCORE: the score-only launches (vd_score, vd_score_ex:
+// mean, scores and sigma, nothing evicted), instantiated with DECODE set
+// and their own ring and occupancy.
+template <int VAR, bool DECODE, bool HF, bool FUSED, bool SCORE = false>
+__global__ void __launch_bounds__(kThreads, SCORE    ? VD_SCORE_MIN_CTAS
+                                            : DECODE ? VD_DECODE_MIN_CTAS
+                                                     : VD_BLOCK_MIN_CTAS)
     evict_kernel(const EvictArgs a) {
+  static_assert(!SCORE || (DECODE && !HF && !FUSED), "score-only instantiation");
   extern __shared__ __align__(16) unsigned char smem_raw[];
   Smem& S = *reinterpret_cast<Smem*>(smem_raw);
-  using Ring = RingShape<DECODE ? DecodeRing::kStages : BlockRing::kStages,
-                         DECODE ? DecodeRing::kItems : BlockRing::kItems>;
+  using Ring = RingShape<SCORE ? ScoreRing::kStages : DECODE ? DecodeRing::kStages
+                                                             : BlockRing::kStages,
+                         SCORE ? ScoreRing::kItems : DECODE ? DecodeRing::kItems
+                                                            : BlockRing::kItems>;
+  constexpr bool score_only = SCORE;
   const int C = a.cluster;
-  const bool with_select = !DECODE && !a.score_only;
-  const SmemLayout L = smem_layout(a.capacity, C, with_select);
+  // score-only at head dims 64, 128, 256 (L2, Norm): the bulk-copy ring
+  const bool bulk = SCORE && score_bulk(VAR, a.d);
+  const int kind = SCORE ? (bulk ? kKindScoreBulk : kKindScore) : DECODE ? kKindDecode : kKindBlock;
+  const SmemLayout L = smem_layout(a.capacity, C, kind);
   const uint32_t ring = smem_addr(smem_raw + L.ring);
   uint32_t* keys = reinterpret_cast<uint32_t*>(smem_raw + L.keys);
   uint16_t* perm = reinterpret_cast<uint16_t*>(smem_raw + L.perm);
@@ -843,20 +1036,24 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
   };
 
   // ---- validation: uniform across the cluster (per-sequence values only) ---
-  if (len0 < 0 || n > a.capacity || (a.mu_running && !a.score_only && a.B > n)) {
+  if (len0 < 0 || n > a.capacity || (a.mu_running && !score_only && a.B > n)) {
     if (rank == 0 && tid == 0) record_status(a.status, kStDeviceLen);
     return;
   }
-  if (!a.score_only && (Nb < 1 || Nb > a.N)) {
+  if (!score_only && (Nb < 1 || Nb > a.N)) {
     if (rank == 0 && tid == 0) record_status(a.status, kStDeviceBudget);
     return;
   }
-  const bool evict = !a.score_only && n > Nb;
+  const bool evict = !score_only && n > Nb;
   if (DECODE && evict && n > Nb + 1) {
     if (rank == 0 && tid == 0) record_status(a.status, kStDeviceBudget);
     return;
   }
-  if (a.score_only && n == 0) return;
+  if (score_only && n == 0) return;
+  BulkRing br{0u, 0u, 0};
+  if constexpr (SCORE) {
+    if (bulk) br = bulk_ring_init(ring, S);
+  }
 
   // column slice of [K | V] this CTA compacts; the running sum is kept for
   // the part of it that lies in the scored tensor (V, or K for the key-side
@@ -872,11 +1069,11 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
   // hole-fill layout: token positions (rows at or above first_new are the
   // appended ones, numbered from pos_new)
   constexpr bool hf = HF;
-  int32_t* posu = hf && !a.score_only ? a.pos + (size_t)u * a.capacity : nullptr;
-  const int pnew = hf && !a.score_only ? a.pos_new[seq] : 0;
+  int32_t* posu = hf && !score_only ? a.pos + (size_t)u * a.capacity : nullptr;
+  const int pnew = hf && !score_only ? a.pos_new[seq] : 0;
   auto pos_of = [&](int r) -> int { return r < first_new ? posu[r] : pnew + (r - first_new); };
 
-  if (!evict && !a.score_only) {
+  if (!evict && !score_only) {
     if (fused) copy_new_rows(kb, vb, knu, vnu, d, chunk0, cps, first_stage, a.B);
     if (hf && rank == 0)
       for (int r = max(first_new, 0) + tid; r < n; r += kThreads) posu[r] = pnew + (r - first_new);
@@ -918,12 +1115,20 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
     // the running sum is loaded before the row sum, whose latency hides it
     const double rs_own = run && tid < d ? a.running_sum[(size_t)u * d + tid] : 0.0;
     const uint16_t* pb = srange(p0, cnt);  // nullptr only where the range straddles
-    sum_rows<Ring, kPackedSum>(0, d8, lpr, cnt,
-                   [&](int i) -> const uint16_t* {
-                     if constexpr (FUSED) return pb ? pb + (size_t)i * d : srow(p0 + i);
-                     else return pb + (size_t)i * d;
-                   },
-                   [](int) { return 1.f; }, S, ring);
+    bool summed = false;
+    if constexpr (SCORE) {
+      if (bulk) {  // score-only rows are never staged: one contiguous range
+        sum_rows_bulk(br, pb, cnt, d, lpr, S, a.status);
+        summed = true;
+      }
+    }
+    if (!summed)
+      sum_rows<Ring, kPackedSum>(0, d8, lpr, cnt,
+                     [&](int i) -> const uint16_t* {
+                       if constexpr (FUSED) return pb ? pb + (size_t)i * d : srow(p0 + i);
+                       else return pb + (size_t)i * d;
+                     },
+                     [](int) { return 1.f; }, S, ring);
     if (C > 1) cluster_sync(); else __syncthreads();
     if (tid < d) {
       ff t{0.f, 0.f};
@@ -960,7 +1165,7 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
   }
   // vd_score reads peer partial sums above and nothing after: release that
   // barrier phase now, wait for it before exiting (peers may still be reading)
-  const bool score_split = C > 1 && a.score_only && VAR != 2;
+  const bool score_split = C > 1 && score_only && VAR != 2;
   if (score_split) cluster_arrive();
 
   // ---- 2. scores -------------------------------------------------------
@@ -1003,7 +1208,7 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
         ff_accumulate(dq_hi, dq_lo, q2);
         dq_lo += fmaf(s, s, -q2);
       }
-      if (!a.score_only) {
+      if (!score_only) {
         bool bad;
         const uint32_t key = score_key(s, bad);
         if (bad) record_status(a.status, kStNonfinite);
@@ -1034,6 +1239,13 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
       const int c_end = min(r1, max(r0, first_stage));
       auto run = [&](auto lanes) {
         constexpr int LPR = decltype(lanes)::value;
+        if constexpr (SCORE) {
+          if (bulk) {
+            score_rows_bulk<VAR, LPR>(br, sb + (size_t)r0 * d, r1 - r0, S.mu, S.mulo, finish_row,
+                                      a.status);
+            return;
+          }
+        }
         if (r1 > c_end)
           score_rows_fast<VAR, LPR, Ring, kScoreBatch>(
               snu + (size_t)(c_end - first_stage) * d, r1 - c_end, S.mu, S.mulo,
@@ -1109,7 +1321,7 @@ __global__ void __launch_bounds__(kThreads, DECODE ? VD_DECODE_MIN_CTAS : VD_BLO
     if constexpr (VAR == 0) {
       if (disp) disp_reduce_cta(ds_hi, ds_lo, dq_hi, dq_lo, S.dsc, S);
     }
-    if (a.score_only) {
+    if (score_only) {
       if (score_split) cluster_wait();
       if constexpr (VAR == 0) {
         if (disp) {

@@ -26,4 +26,8 @@ const void* small_kernel_dir(bool decode, bool fused) {
        reinterpret_cast<const void*>(&small_evict_kernel<1, true, true>)}};
   return k[decode][fused];
 }
+
+const void* score_kernel_dir() {
+  return reinterpret_cast<const void*>(&evict_kernel<1, true, false, false, true>);
+}
 }  // namespace vd

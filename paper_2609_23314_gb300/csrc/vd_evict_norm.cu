@@ -26,4 +26,8 @@ const void* small_kernel_norm(bool decode, bool fused) {
        reinterpret_cast<const void*>(&small_evict_kernel<2, true, true>)}};
   return k[decode][fused];
 }
+
+const void* score_kernel_norm() {
+  return reinterpret_cast<const void*>(&evict_kernel<2, true, false, false, true>);
+}
 }  // namespace vd
