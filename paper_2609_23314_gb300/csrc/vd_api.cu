@@ -406,19 +406,22 @@ bool cached_fits(const void* kern, long long groups, int c, size_t smem, DeviceS
 }
 
 vd_status launch(const void* kern, long long groups, int c, size_t smem, const void* params,
-                 cudaStream_t s) {
+                 cudaStream_t s, bool dependent = false) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3((unsigned)(groups * c));
   cfg.blockDim = dim3(kThreads);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = s;
-  cudaLaunchAttribute attr;
-  attr.id = cudaLaunchAttributeClusterDimension;
-  attr.val.clusterDim.x = (unsigned)c;
-  attr.val.clusterDim.y = 1;
-  attr.val.clusterDim.z = 1;
-  cfg.attrs = &attr;
-  cfg.numAttrs = 1;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = (unsigned)c;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  // a programmatic dependent launch (the kernel waits in griddepcontrol.wait)
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = dependent ? 2 : 1;
   void* args[] = {const_cast<void*>(params)};
   if (cudaLaunchKernelExC(&cfg, kern, args) != cudaSuccess) {
     cudaGetLastError();
@@ -503,7 +506,7 @@ vd_status run(const vd_cache* c, int32_t N, const int32_t* N_dev, int32_t B, vd_
     a.cluster = a.units_per_seq;
     if (cached_fits(sk, c->n_seq, a.cluster, ssmem, *st)) {
       const vd::SmallArgs sa{a, (int32_t)units};
-      return launch(sk, c->n_seq, a.cluster, ssmem, &sa, s);
+      return launch(sk, c->n_seq, a.cluster, ssmem, &sa, s, true);
     }
   }
   size_t smem = 0;

@@ -144,6 +144,23 @@ __device__ __forceinline__ void st16(void* p, const uint4& v) {
 }
 
 // ---------------------------------------------------------------------------
+// Programmatic dependent launch.  A kernel launched with programmatic stream
+// serialization may start before the previous kernel on its stream has
+// finished; griddepcontrol.wait blocks until that kernel has completed and
+// its memory is visible (a no-op for a normal launch), so it must come before
+// the first access to memory.  launch_dependents lets the next kernel on the
+// stream, if it was launched the same way, be scheduled once every CTA of
+// this grid has issued it (it then waits in its own griddepcontrol.wait).
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ void grid_dependency_wait() {
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+}
+
+__device__ __forceinline__ void grid_launch_dependents() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
+// ---------------------------------------------------------------------------
 // Bulk copies: one thread moves a contiguous block of global memory into this
 // CTA's own shared memory (cp.async.bulk, no multicast; both addresses and the
 // size multiples of 16 bytes), and the copy's completion is counted on an

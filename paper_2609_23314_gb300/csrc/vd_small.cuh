@@ -99,6 +99,10 @@ struct SmallArgs {
 template <int VAR, bool DECODE, bool FUSED>
 __global__ void __launch_bounds__(kThreads, 1) small_evict_kernel(const SmallArgs sa) {
   const EvictArgs& a = sa.e;
+  // launched as a programmatic dependent: wait for the previous kernel on the
+  // stream before reading anything, and let the next one be scheduled
+  grid_dependency_wait();
+  grid_launch_dependents();
   extern __shared__ __align__(16) unsigned char smem_raw[];
   SmallSmem& S = *reinterpret_cast<SmallSmem*>(smem_raw);
   const int d = a.d, d8 = d >> 3, cap = a.capacity;
