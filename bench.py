@@ -171,7 +171,8 @@ def ncu_traffic(workload: str, layout: str = "ordered", separate: bool = False,
         with open(path) as f:
             t = json.load(f)
         key = workload if layout == "ordered" else f"{workload}:{layout}"
-        e = t[key + (":separate" if separate else "")]
+        key += (":separate" if separate else "") + (":recompute" if mu == "recompute" else "")
+        e = t[key]
         if e.get("source_hash") != kernel_source_hash():
             return None
         for field, want in (("kernel", kernel), ("units", units), ("mu", mu)):
@@ -925,6 +926,7 @@ def measure_dispersion(args, device, variant, peak, rank):
 
     ms_re = timed(vd.VD_MU_RECOMPUTE)
     ms = timed(vd.VD_MU_RUNNING)
+    kernel = "vd::evict_kernel<0, true, false, false, true> (score only)"
     # the realized sigma_V / sigma_K of the generator (untimed)
     sigma_k = torch.empty_like(sigma)
     vd.vd_score_ex(w.cache, vd.VD_SCORE_L2, True, None, sigma_k)
@@ -932,15 +934,18 @@ def measure_dispersion(args, device, variant, peak, rank):
     n = int(w.cache.len[0])
     alg = w.U * n * w.d * 2 + w.U * 4
     achieved = alg / (ms / 1e3) / 1e9
+    tr = ncu_traffic("prefill_wide:sigma", kernel=kernel, units=w.U, mu="running")
+    tr_re = ncu_traffic("prefill_wide:sigma", kernel=kernel, units=w.U, mu="recompute")
     res = {"value": w.U * n / (ms / 1e3), "step_ms": ms, "mean": "running sum",
            "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
-                        "frac": achieved / peak, "kernel": "vd::evict_kernel<0, true, false, false> (score only)",
+                        "frac": achieved / peak, "kernel": kernel, "traffic": tr,
                         "algorithmic_bytes_per_launch": alg, "kernel_ms": ms,
                         "sigma_v_mean": float(sigma.mean().item()),
                         "sigma_k_mean": float(sigma_k.mean().item()),
                         "sigma_v_over_sigma_k": ratio},
            "recomputed_mean": {"value": w.U * n / (ms_re / 1e3), "step_ms": ms_re,
                                "frac_of_peak": alg / (ms_re / 1e3) / 1e9 / peak,
+                               "traffic": tr_re,
                                "note": "V read twice (sum, then scores); frac counts it once"}}
     del w
     torch.cuda.empty_cache()
@@ -1161,6 +1166,13 @@ def run_vd(args):
                           round(tr / rf["algorithmic_bytes_per_launch"], 3) if tr else None,
                           round(r["e2e"]["value"] / 1e9, 3)]
 
+    if args.dispersion_only:
+        # the sigma pass alone (score-only launches, both mean modes): a short
+        # run whose launches come in a fixed order, for profiling
+        disp = measure_dispersion(args, device, variant, peak, rank)
+        if rank == 0:
+            print(json.dumps({"metric": METRIC, "unit": UNIT, "dispersion": disp}), flush=True)
+        return
     primary = one(args.workload, args.steps, args.layout)
     summarize(f"{args.workload} ({primary['config']['mu']} mean)", primary)
     base = None
@@ -1240,10 +1252,14 @@ def run_vd(args):
         disp = measure_dispersion(args, device, variant, peak, rank)
         stricter(disp["roofline"], read_gbs)
         extensions["dispersion"] = disp
+        alg_d = disp["roofline"]["algorithmic_bytes_per_launch"]
+        tr_d, tr_r = disp["roofline"]["traffic"], disp["recomputed_mean"]["traffic"]
         summary["sigma pass (running, recomputed mean)"] = [
             round(disp["step_ms"], 4), round(disp["roofline"]["frac"], 3),
+            round(tr_d / alg_d, 3) if tr_d else None,
             round(disp["recomputed_mean"]["step_ms"], 4),
-            round(disp["recomputed_mean"]["frac_of_peak"], 3)]
+            round(disp["recomputed_mean"]["frac_of_peak"], 3),
+            round(tr_r / alg_d, 3) if tr_r else None]
     if rank == 0:
         line = {
             "metric": METRIC, "value": primary["value"], "unit": UNIT, "n_gpus": ws,
@@ -1370,6 +1386,8 @@ def main(argv=None):
     ap.add_argument("--n-seq", type=int, default=None,
                     help="override the workload's number of sequences (smaller profiling cases)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--dispersion-only", action="store_true",
+                    help="time only the sigma pass of the workload (profiling runs)")
     args = ap.parse_args(argv)
     if args.warmup < 3:
         ap.error("--warmup must be at least 3")

@@ -98,7 +98,10 @@ def test_traffic_is_reported_only_for_the_captured_sources(monkeypatch):
                              mu=e["mu"]) == e["dram_bytes_per_launch"]
     assert bench.ncu_traffic("prefill_wide", units=e["units"] // 2) is None
     assert bench.ncu_traffic("prefill_wide", kernel=e["kernel"].replace("<0,", "<1,")) is None
-    assert bench.ncu_traffic("prefill_wide", mu="recompute") is None
+    # the recomputed mean has an entry of its own
+    r = t["prefill_wide:recompute"]
+    assert bench.ncu_traffic("prefill_wide", mu="recompute") == r["dram_bytes_per_launch"]
+    assert r["mu"] == "recompute" and r["dram_bytes_per_launch"] != e["dram_bytes_per_launch"]
     monkeypatch.setattr(bench, "kernel_source_hash", lambda: "changed")
     assert bench.ncu_traffic("prefill_wide") is None
 
