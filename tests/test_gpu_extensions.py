@@ -337,3 +337,23 @@ def test_option_errors():
     attn[..., 3] = 1.0                        # a weight of 1: infinite factor
     vd.vd_evict_block_ex(cache, 32, attn=attn)
     assert vd.vd_get_device_status() == 4
+
+
+@pytest.mark.parametrize("var", [oracle.L2, oracle.NORM], ids=["l2", "norm"])
+@pytest.mark.parametrize("d", [64, 128, 256])
+@pytest.mark.parametrize("cluster", [1, 2, 4])
+def test_score_only_bulk_ring_matches_the_eviction_score_pass(var, d, cluster, monkeypatch):
+    """vd_score at head dims 64/128/256 streams its rows through bulk copies;
+    the eviction kernel streams them through per-thread asynchronous copies.
+    With the same cluster size (so each CTA sums and scores the same rows)
+    the mean and every score are bit-identical."""
+    monkeypatch.setenv("VD_CLUSTER_SIZE", str(cluster))
+    n = 1500                                   # several 32 KB stages and a ragged last one
+    cache = filled(2, 2, 2, n, d, [n, n - 333], seed=91 + d)
+    sc = torch.full(cache.unit_shape() + (n,), float("nan"), device="cuda")
+    vd.vd_score(cache, var, sc)
+    ev = vd.Cache(cache.k.clone(), cache.v.clone(), cache.len.clone())
+    sc2 = torch.full_like(sc, float("nan"))
+    vd.vd_evict_block(ev, n - 400, None, 0, var, vd.VD_MU_RECOMPUTE, None, None, sc2)
+    assert vd.vd_get_device_status() == 0
+    assert torch.equal(sc.nan_to_num(-1.0), sc2.nan_to_num(-1.0))
