@@ -217,3 +217,32 @@ def test_decode_over_budget_and_bad_length():
     vd.vd_evict_block(cache, N, None, 0, oracle.L2, vd.VD_MU_RECOMPUTE, None, None, None)
     assert vd.vd_get_device_status() == 7   # VD_ERR_DEVICE_LEN (sequence 0)
     assert cache.len.tolist() == [N + 6, N]
+
+
+@pytest.mark.parametrize("var", VARS, ids=VAR_IDS)
+def test_head_dim_256(orc, var):
+    """The widest head dim: 4 * capacity * 256 <= 64 KB leaves 64 rows."""
+    d, cap, N, B = 256, 64, 40, 24
+    cache = filled_cache(2, 1, 3, cap, d, [cap, N + 5], seed=81)
+    evict_and_check(orc, cache, N, B, var, vd.VD_MU_RECOMPUTE)
+
+
+def test_nan_row_is_reported_and_evicted_first(orc):
+    """A NaN in one row makes its Norm score NaN (the Norm rule reads no
+    mean, so the other rows keep finite scores): the event is still run, the
+    status reports VD_ERR_NONFINITE, and that row is evicted before any
+    other (NaN ranks lowest), as in the oracle."""
+    d, n, N = 64, 100, 99
+    cache = filled_cache(1, 1, 2, n, d, [n], seed=83)
+    cache.v[0, 0, 0, 37, 5] = float("nan")
+    kept = torch.full(cache.unit_shape() + (N,), -7, dtype=torch.int32, device="cuda")
+    pre_v = bits(units_view(cache.v))
+    vd.vd_evict_block(cache, N, None, 0, oracle.NORM, vd.VD_MU_RECOMPUTE, None, kept, None)
+    assert vd.vd_get_device_status() == 4   # VD_ERR_NONFINITE
+    kh = kept.view(2, N).cpu().numpy()
+    assert 37 not in kh[0].tolist()          # the NaN row went
+    # unit 1 has no NaN: it evicts its lowest score, as the oracle does
+    s0 = orc.scores(pre_v[0, :n], oracle.NORM)
+    assert np.isnan(s0[37]) and np.array_equal(kh[0], orc.select_top_n(s0, N))
+    s1 = orc.scores(pre_v[1, :n], oracle.NORM)
+    assert np.array_equal(kh[1], orc.select_top_n(s1, N))
