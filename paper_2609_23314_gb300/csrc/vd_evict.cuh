@@ -974,6 +974,74 @@ __device__ __forceinline__ void move_rows(uint16_t* kb, uint16_t* vb, int d, int
   }
 }
 
+// move_rows through this CTA's cp.async ring (block hole-fill events, which
+// move up to B rows): item i of the h * cps (row, chunk) items is copied from
+// row src_of(i / cps) to row dst_of(i / cps) of the column slice.  Sources
+// lie at or above N and destinations below it, so no copy can read what
+// another writes: each thread stores what it loaded itself, with no barrier
+// between tiles, and keeps kStages x kItems copies in flight.  A row
+// outside [0, n) is skipped and recorded as kStInternal.
+template <class Ring, class SrcOf, class DstOf>
+__device__ __forceinline__ void move_rows_ring(uint16_t* kb, uint16_t* vb, int d, int chunk0,
+                                               int cps, int h, int n, SrcOf src_of, DstOf dst_of,
+                                               unsigned* status, const uint16_t* kn,
+                                               const uint16_t* vn, int first_stage,
+                                               uint32_t ring) {
+  constexpr int kStages = Ring::kStages, kItems = Ring::kItems;
+  const int d8 = d >> 3;
+  const int items = h * cps;
+  const int per_stage = kThreads * kItems;
+  const int nst = (items + per_stage - 1) / per_stage;
+  const uint32_t my = ring + (uint32_t)threadIdx.x * 16u;
+  auto slot = [&](int st, int u) {
+    return my + (uint32_t)((st * kItems + u) * kThreads * 16);
+  };
+  // item of this thread's u-th copy of stage st, and its destination
+  auto item_of = [&](int st, int u) { return (st * kItems + u) * kThreads + (int)threadIdx.x; };
+  auto dst_ptr = [&](int it) -> uint16_t* {
+    const int i = it / cps, c = chunk0 + it % cps;
+    const int dr = dst_of(i), sr = src_of(i);
+    if ((unsigned)sr >= (unsigned)n || (unsigned)dr >= (unsigned)n) return nullptr;
+    return (c < d8 ? kb + c * 8 : vb + (c - d8) * 8) + (size_t)dr * d;
+  };
+  auto issue = [&](int st) {
+    if (st < nst) {
+#pragma unroll
+      for (int u = 0; u < kItems; ++u) {
+        const int it = item_of(st, u);
+        if (it < items) {
+          const int i = it / cps, c = chunk0 + it % cps;
+          const int sr = src_of(i), dr = dst_of(i);
+          if ((unsigned)sr < (unsigned)n && (unsigned)dr < (unsigned)n) {
+            const uint16_t* sp = sr >= first_stage
+                                     ? (c < d8 ? kn + c * 8 : vn + (c - d8) * 8) +
+                                           (size_t)(sr - first_stage) * d
+                                     : (c < d8 ? kb + c * 8 : vb + (c - d8) * 8) + (size_t)sr * d;
+            cp_async16(slot(st % kStages, u), sp);
+          } else {
+            record_status(status, kStInternal);
+          }
+        }
+      }
+    }
+    cp_async_commit();
+  };
+  for (int st = 0; st < kStages; ++st) issue(st);
+  for (int st = 0; st < nst; ++st) {
+    cp_async_wait<kStages - 1>();
+#pragma unroll 1
+    for (int u = 0; u < kItems; ++u) {
+      const int it = item_of(st, u);
+      if (it < items) {
+        uint16_t* dp = dst_ptr(it);
+        if (dp) st16(dp, ld_shared16(slot(st % kStages, u)));
+      }
+    }
+    issue(st + kStages);
+  }
+  cp_async_wait<0>();
+}
+
 // VAR: 0 L2, 1 Dir, 2 Norm.  DECODE: one-token eviction (arg-min) instead of
 // the radix select.  HF: hole-fill layout (compiled separately, so the ordered
 // layout carries none of its code).  FUSED: the new rows are read from the
@@ -1503,7 +1571,11 @@ __global__ void __launch_bounds__(kThreads, SCORE    ? VD_SCORE_MIN_CTAS
       copy_new_rows(kb, vb, knu, vnu, d, chunk0, cps, first_stage, Nb - first_stage);
       __syncthreads();
     }
-    move_rows(kb, vb, d, chunk0, cps, h, n, src, dst, a.status, knu, vnu, first_stage);
+    if constexpr (DECODE)
+      move_rows(kb, vb, d, chunk0, cps, h, n, src, dst, a.status, knu, vnu, first_stage);
+    else
+      move_rows_ring<Ring>(kb, vb, d, chunk0, cps, h, n, src, dst, a.status, knu, vnu,
+                           first_stage, ring);
     if (rank == 0) {
       for (int r = max(first_new, 0) + tid; r < Nb; r += kThreads) posu[r] = pnew + (r - first_new);
       int32_t* ko = a.kept_out ? a.kept_out + (size_t)u * a.N : nullptr;
