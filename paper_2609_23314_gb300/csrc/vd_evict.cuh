@@ -699,18 +699,23 @@ struct Selection {
   int cnt_eq;
 };
 
+// first_ready: S.hist[0] already holds this CTA's counts of the keys' top
+// byte (built by the score pass), so the first pass skips its counting loop.
 template <class KeyOf>
 __device__ __forceinline__ Selection cluster_radix_select(KeyOf key_of, int R, int N, int C,
-                                                          Smem& S) {
+                                                          Smem& S, bool first_ready = false) {
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   uint32_t prefix = 0, pmask = 0;
   int need = N, cnt = 0;
   for (int pass = 0; pass < 4; ++pass) {
     const int shift = 24 - 8 * pass;
     uint32_t* h = S.hist[pass & 1];
-    h[tid] = 0;
-    __syncthreads();
-    for (int base = 0; base < R; base += kThreads) {
+    const bool counted = pass == 0 && first_ready;
+    if (!counted) {
+      h[tid] = 0;
+      __syncthreads();
+    }
+    for (int base = 0; !counted && base < R; base += kThreads) {
       const int j = base + tid;
       bool ok = false;
       uint32_t key = 0u;
@@ -1163,6 +1168,13 @@ __global__ void __launch_bounds__(kThreads, SCORE    ? VD_SCORE_MIN_CTAS
     return;
   }
 
+  // block eviction without attention weights: the score pass counts the
+  // keys' top byte for the select's first radix pass as it writes them
+  const bool hist_pre = !DECODE && !score_only && a.weights == nullptr;
+  if (hist_pre) {
+    S.hist[0][tid] = 0;
+    __syncthreads();
+  }
   // ---- 1. mean ---------------------------------------------------------
   const int rows_per = (n + C - 1) / C;
   const int r0 = min(n, (int)rank * rows_per), r1 = min(n, r0 + rows_per);
@@ -1294,6 +1306,7 @@ __global__ void __launch_bounds__(kThreads, SCORE    ? VD_SCORE_MIN_CTAS
           }
         } else {
           keys[item] = key;
+          if (hist_pre) atomicAdd(&S.hist[0][key >> 24], 1u);  // the select's first pass
         }
       }
     };
@@ -1477,7 +1490,7 @@ __global__ void __launch_bounds__(kThreads, SCORE    ? VD_SCORE_MIN_CTAS
           ok = true;
           return keys[j];
         },
-        R, Nb, C, S);
+        R, Nb, C, S, hist_pre);
     if constexpr (VAR == 0) {
       if (disp && rank == 0 && tid == 0) a.disp_out[u] = disp_finish(S, C, n);
     }
