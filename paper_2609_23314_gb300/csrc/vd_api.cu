@@ -6,6 +6,7 @@
 // variable: the library allocates no device memory).
 #include <cuda_runtime.h>
 
+#include <algorithm>
 #include <climits>
 #include <cmath>
 #include <cstdint>
@@ -120,6 +121,7 @@ struct ClusterChoice {
   long long units;
   int d, capacity, kind, want, c;  // kind: vd::kKind*, or kFitsKind (cached_fits)
   size_t smem;
+  long long solo, want_solo;       // split launch: units run one CTA each (split_plan)
 };
 constexpr int kChoiceSlots = 32;
 
@@ -331,28 +333,107 @@ int choose_cluster(const void* kern, long long units, int d, int capacity, int k
   return chosen;
 }
 
-// choose_cluster, remembered per launch shape.
+// Split launch, for launches that fit one wave of one CTA per unit and
+// carry more units than the GPU has SMs.  The block scheduler hands CTAs out
+// breadth-first, so with U = k P + L units on P SMs (0 < L < P), L SMs run
+// k + 1 whole units and the rest k, and the launch lasts as long as the
+// busiest SMs (prefill_wide in the hole-fill layout, 336 units on 152 SMs:
+// the CTAs of the 32 SMs that held three finished 28 us after the median).
+// Instead, a first launch runs the first k P units (rounded down to a
+// multiple of c) one CTA each, and a second launch, a programmatic dependent
+// of the first, runs each remaining unit on a cluster of c CTAs: its CTAs
+// take the slots the first leaves free, so an SM carries at most
+// k + ceil(L c / P) / c units.  c in {2, 4, 8, 16} is the one with the
+// smallest such load whose CTAs still form one wave; the split is taken when
+// it lowers the load by at least a quarter of a unit.  Used by hole-fill
+// block eviction and the score-only launches (each reads its units once and
+// moves few rows, so a unit's time is its share of the read bandwidth);
+// VD_SPLIT_LAUNCH=0 turns it off.  Returns the number of units of the first
+// launch (0: no split) and sets *c_out and *smem_out for the second.
+long long split_plan(const void* kern, long long units, int d, int capacity, int kind,
+                     const DeviceState& st, int* c_out, size_t* smem_out) {
+  const long long P = st.sms;
+  if (P < 1 || units <= P) return 0;
+  const size_t smem1 = vd::smem_layout(capacity, 1, kind).total;
+  if (smem1 > (size_t)st.smem_optin) return 0;
+  int occ = 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, kern, kThreads, smem1) != cudaSuccess) {
+    cudaGetLastError();
+    return 0;
+  }
+  if (occ < 1 || units > P * occ) return 0;  // more than one wave: CTAs balance themselves
+  const long long k = units / P;
+  if (units % P == 0) return 0;
+  double best = (double)(k + 1) - 0.25;
+  long long best_solo = 0;
+  for (int c = 2; c <= 16; c *= 2) {
+    if (!cluster_allowed(c, d)) continue;
+    const long long solo = (k * P) / c * c;
+    const long long joint = units - solo;
+    if (solo + joint * c > P * occ) continue;  // one wave
+    const double load = (double)((solo + P - 1) / P) + (double)((joint * c + P - 1) / P) / c;
+    const size_t smem_c = vd::smem_layout(capacity, c, kind).total;
+    if (load < best && cluster_fits(kern, joint, c, smem_c)) {
+      best = load;
+      best_solo = solo;
+      *c_out = c;
+      *smem_out = smem_c;
+    }
+  }
+  return best_solo;
+}
+
+// choose_cluster (and split_plan), remembered per launch shape.  A forced
+// cluster size (VD_CLUSTER_SIZE) turns the automatic split off;
+// VD_SOLO_UNITS with it forces a split whose first launch runs that many
+// units (at most all but one) one CTA each, for tests.
 int cached_cluster(const void* kern, long long units, int d, int capacity, int kind,
-                   bool holefill, DeviceState& st, size_t* smem_out) {
+                   bool holefill, DeviceState& st, size_t* smem_out, long long* solo_out) {
   const char* env = std::getenv("VD_CLUSTER_SIZE");
   const int want = env ? std::atoi(env) : 0;
+  // want_solo: the forced first part (VD_SOLO_UNITS, with a forced cluster
+  // size), else 0 when the split is turned off, else -1 (automatic)
+  long long want_solo = -1;
+  if (want >= 1) {
+    const char* senv = std::getenv("VD_SOLO_UNITS");
+    if (senv) want_solo = std::atoll(senv);
+  } else {
+    const char* off = std::getenv("VD_SPLIT_LAUNCH");
+    if (off && std::atoi(off) == 0) want_solo = 0;
+  }
   {
     std::lock_guard<std::mutex> lk(g_mu);
     for (int i = 0; i < st.n_choice; ++i) {
       const ClusterChoice& e = st.choice[i];
       if (e.kern == kern && e.units == units && e.d == d && e.capacity == capacity &&
-          e.kind == kind && e.want == want) {
+          e.kind == kind && e.want == want && e.want_solo == want_solo) {
         *smem_out = e.smem;
+        *solo_out = e.solo;
         return e.c;
       }
     }
   }
-  const int c = choose_cluster(kern, units, d, capacity, kind, holefill, want, st,
-                               smem_out);
+  int c = choose_cluster(kern, units, d, capacity, kind, holefill, want, st, smem_out);
+  long long solo = 0;
+  if (want >= 1 && want_solo > 0) {
+    solo = std::min(want_solo, units - 1);
+  } else if (want < 1 && want_solo != 0 &&
+             ((kind == vd::kKindBlock && holefill) || kind == vd::kKindScore ||
+              kind == vd::kKindScoreBulk)) {
+    int cs = c;
+    size_t sm = *smem_out;
+    solo = split_plan(kern, units, d, capacity, kind, st, &cs, &sm);
+    if (solo > 0) {
+      c = cs;
+      *smem_out = sm;
+    }
+  }
   std::lock_guard<std::mutex> lk(g_mu);
-  st.choice[st.next_choice] = ClusterChoice{kern, units, d, capacity, kind, want, c, *smem_out};
+  st.choice[st.next_choice] =
+      ClusterChoice{kern, units, d, capacity, kind, want, c, *smem_out, solo, want_solo};
   st.next_choice = (st.next_choice + 1) % kChoiceSlots;
   if (st.n_choice < kChoiceSlots) ++st.n_choice;
+  *solo_out = solo;
   return c;
 }
 
@@ -399,7 +480,8 @@ bool cached_fits(const void* kern, long long groups, int c, size_t smem, DeviceS
   }
   const bool fits = c == 1 || cluster_fits(kern, groups, c, smem);
   std::lock_guard<std::mutex> lk(g_mu);
-  st.choice[st.next_choice] = ClusterChoice{kern, groups, 0, 0, kFitsKind, c, fits ? c : 0, smem};
+  st.choice[st.next_choice] =
+      ClusterChoice{kern, groups, 0, 0, kFitsKind, c, fits ? c : 0, smem, 0, 0};
   st.next_choice = (st.next_choice + 1) % kChoiceSlots;
   if (st.n_choice < kChoiceSlots) ++st.n_choice;
   return fits;
@@ -498,6 +580,7 @@ vd_status run(const vd_cache* c, int32_t N, const int32_t* N_dev, int32_t B, vd_
   a.disp_out = disp_out;
   a.k_new = static_cast<const uint16_t*>(k_new);
   a.v_new = static_cast<const uint16_t*>(v_new);
+  a.unit_base = 0;
   if (use_small(c, score_only, holefill, weights, disp_out, score_k, *st)) {
     // one launch: the kernel also sets the sequences' lengths
     // grid: n_seq clusters of units_per_seq CTAs, one CTA per unit
@@ -510,10 +593,38 @@ vd_status run(const vd_cache* c, int32_t N, const int32_t* N_dev, int32_t B, vd_
     }
   }
   size_t smem = 0;
-  a.cluster = cached_cluster(kern, units, c->head_dim, c->capacity, kind, holefill, *st, &smem);
+  long long solo = 0;
+  a.cluster =
+      cached_cluster(kern, units, c->head_dim, c->capacity, kind, holefill, *st, &smem, &solo);
   if (smem > (size_t)st->smem_optin) return VD_ERR_UNSUPPORTED;
 
-  r = launch(kern, units, a.cluster, smem, &a, s);
+  if (solo > 0) {
+    // split launch: units [0, solo) one CTA each, then the rest on clusters,
+    // as a programmatic dependent of the first part
+    vd::EvictArgs a1 = a;
+    a1.cluster = 1;
+    const size_t smem1 = vd::smem_layout(c->capacity, 1, kind).total;
+    if (smem1 > (size_t)st->smem_optin) return VD_ERR_UNSUPPORTED;
+    r = launch(kern, solo, 1, smem1, &a1, s);
+    if (r != VD_OK) return r;
+    // the second part's per-unit pointers start at unit `solo`
+    const size_t rows = (size_t)solo * c->capacity, dd = (size_t)c->head_dim;
+    a.unit_base = (int32_t)solo;
+    a.k += rows * dd;
+    a.v += rows * dd;
+    if (a.running_sum) a.running_sum += (size_t)solo * dd;
+    if (a.kept_out) a.kept_out += (size_t)solo * a.N;
+    if (a.evicted_out) a.evicted_out += solo;
+    if (a.scores_out) a.scores_out += rows;
+    if (a.pos) a.pos += rows;
+    if (a.weights) a.weights += rows;
+    if (a.disp_out) a.disp_out += solo;
+    if (a.k_new) a.k_new += (size_t)solo * a.B * dd;
+    if (a.v_new) a.v_new += (size_t)solo * a.B * dd;
+    r = launch(kern, units - solo, a.cluster, smem, &a, s, true);
+  } else {
+    r = launch(kern, units, a.cluster, smem, &a, s);
+  }
   if (r != VD_OK || score_only) return r;
   const int threads = 256;
   vd_len_clamp_kernel<<<(c->n_seq + threads - 1) / threads, threads, 0, s>>>(

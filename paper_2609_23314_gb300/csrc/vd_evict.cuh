@@ -166,6 +166,10 @@ struct EvictArgs {
   // (nullable: the rows were appended beforehand)
   const uint16_t* k_new;
   const uint16_t* v_new;
+  // split launch (two launches over disjoint units): the units before this
+  // launch's first one.  Only the sequence index adds it; every per-unit
+  // pointer above comes offset to the launch's first unit.
+  int32_t unit_base;
 };
 
 // Fixed part of the dynamic shared memory.  After it (16-byte aligned): the
@@ -1054,11 +1058,8 @@ __device__ __forceinline__ void move_rows_ring(uint16_t* kb, uint16_t* vb, int d
 // of that code.  SCORE: the score-only launches (vd_score, vd_score_ex:
 // mean, scores and sigma, nothing evicted), instantiated with DECODE set
 // and their own ring and occupancy.
-template <int VAR, bool DECODE, bool HF, bool FUSED, bool SCORE = false>
-__global__ void __launch_bounds__(kThreads, SCORE    ? VD_SCORE_MIN_CTAS
-                                            : DECODE ? VD_DECODE_MIN_CTAS
-                                                     : VD_BLOCK_MIN_CTAS)
-    evict_kernel(const EvictArgs a) {
+template <int VAR, bool DECODE, bool HF, bool FUSED, bool SCORE>
+__device__ __forceinline__ void evict_unit(const EvictArgs& a) {
   static_assert(!SCORE || (DECODE && !HF && !FUSED), "score-only instantiation");
   extern __shared__ __align__(16) unsigned char smem_raw[];
   Smem& S = *reinterpret_cast<Smem*>(smem_raw);
@@ -1080,7 +1081,7 @@ __global__ void __launch_bounds__(kThreads, SCORE    ? VD_SCORE_MIN_CTAS
   const unsigned rank = C > 1 ? cluster_ctarank() : 0u;
   const int u = C > 1 ? (int)cluster_id_x() : (int)blockIdx.x;
   const int d = a.d, d8 = d >> 3;
-  const int seq = u / a.units_per_seq;
+  const int seq = (u + a.unit_base) / a.units_per_seq;  // unit pointers come pre-offset
   constexpr bool fused = FUSED;  // the new rows are still in the staging buffers
   // packed-pair row sums everywhere but the Dir block kernels (register budget)
   constexpr bool kPackedSum = !(VAR == 1 && !DECODE);
@@ -1605,6 +1606,24 @@ __global__ void __launch_bounds__(kThreads, SCORE    ? VD_SCORE_MIN_CTAS
   }
 
   if (DECODE && C > 1) cluster_wait();
+}
+
+// One unit per cluster of C CTAs (evict_unit).  Split launches (the host's
+// split_plan) run the units in two launches on one stream, the second a
+// programmatic dependent launch whose CTAs take the slots the first leaves
+// free.  So every kernel lets its dependents be scheduled at once.  The two
+// parts touch disjoint units, so the second reads nothing the first writes;
+// it waits for the first only before it ends (griddepcontrol.wait, a no-op
+// in a normal launch), so that work queued after it on the stream also
+// follows the first.
+template <int VAR, bool DECODE, bool HF, bool FUSED, bool SCORE = false>
+__global__ void __launch_bounds__(kThreads, SCORE    ? VD_SCORE_MIN_CTAS
+                                            : DECODE ? VD_DECODE_MIN_CTAS
+                                                     : VD_BLOCK_MIN_CTAS)
+    evict_kernel(const EvictArgs a) {
+  grid_launch_dependents();
+  evict_unit<VAR, DECODE, HF, FUSED, SCORE>(a);
+  grid_dependency_wait();
 }
 
 }  // namespace vd
