@@ -189,6 +189,8 @@ struct Smem {
   unsigned long long best;  // decode: this CTA's (key, -tie-break) minimum
   unsigned long long wbest[kWarps];
   int sel_digit, sel_above, sel_cnt;
+  uint32_t sel_t;  // rank resolution: the threshold key
+  int ncand;       // rank resolution: this CTA's candidates (in ghist, read by peers)
   int cnt_gt, cnt_eq;  // this CTA's keys > t and == t (read by peers)
   int mu_zero;
   int best_slot;       // hole-fill decode: the slot of `best`
@@ -705,6 +707,15 @@ struct Selection {
 
 // first_ready: S.hist[0] already holds this CTA's counts of the keys' top
 // byte (built by the score pass), so the first pass skips its counting loop.
+//
+// As soon as a pass leaves at most kThreads keys in the cluster that share
+// the threshold's prefix (the candidates), the remaining passes are replaced
+// by ranking the candidates directly: every CTA compacts its own candidates
+// (into ghist, which peers then read), gathers the cluster's candidates, and
+// each thread counts how many candidates are greater than and equal to its
+// own.  The threshold is the candidate with g < need <= g + e.  Candidate
+// counts come from the cluster-summed histogram, so every CTA of the cluster
+// takes the same branch.
 template <class KeyOf>
 __device__ __forceinline__ Selection cluster_radix_select(KeyOf key_of, int R, int N, int C,
                                                           Smem& S, bool first_ready = false) {
@@ -778,6 +789,59 @@ __device__ __forceinline__ Selection cluster_radix_select(KeyOf key_of, int R, i
     prefix |= (uint32_t)S.sel_digit << shift;
     pmask |= 255u << shift;
     cnt = S.sel_cnt;
+    if (pass == 3 || cnt > kThreads) continue;
+
+    // ---- rank resolution among the cnt candidates -------------------------
+    // (ghist is free once every thread has read the scan's result above)
+    if (tid == 0) S.ncand = 0;
+    __syncthreads();
+    for (int base = 0; base < R; base += kThreads) {
+      const int j = base + tid;
+      bool ok = false;
+      uint32_t key = 0u;
+      if (j < R) key = key_of(j, ok);
+      const bool match = ok && (key & pmask) == prefix;
+      const unsigned act = __ballot_sync(kFull, match);
+      int at = 0;
+      if (lane == 0 && act) at = atomicAdd(&S.ncand, __popc(act));
+      at = __shfl_sync(kFull, at, 0);
+      if (match) S.ghist[at + __popc(act & ((1u << lane) - 1u))] = key;
+    }
+    if (C > 1) cluster_sync(); else __syncthreads();
+    // every CTA gathers the cluster's candidates, in rank order, into the
+    // histogram buffer that no peer reads any more (the other pass's)
+    uint32_t* all = S.hist[(pass + 1) & 1];
+    uint32_t mine = 0u;
+    {
+      int off = 0;
+      for (int rr = 0; rr < C; ++rr) {
+        const int nc = C > 1 ? (int)ld_cluster_u32(mapa(smem_addr(&S.ncand), (unsigned)rr))
+                             : S.ncand;
+        if (tid >= off && tid < off + nc)
+          mine = C > 1 ? ld_cluster_u32(mapa(smem_addr(&S.ghist[tid - off]), (unsigned)rr))
+                       : S.ghist[tid - off];
+        off += nc;
+      }
+    }
+    if (tid < cnt) all[tid] = mine;
+    __syncthreads();
+    if (tid < cnt) {
+      int g = 0, e = 0;
+      for (int i = 0; i < cnt; ++i) {
+        const uint32_t o = all[i];
+        g += o > mine;
+        e += o == mine;
+      }
+      if (g < need && need <= g + e) {  // every candidate equal to t writes the same
+        S.sel_t = mine;
+        S.sel_above = need - g;
+        S.sel_cnt = e;
+      }
+    }
+    __syncthreads();
+    // peers read this CTA's candidates (ghist) until they pass the caller's
+    // next cluster barrier; nothing writes ghist before it
+    return {S.sel_t, S.sel_above, S.sel_cnt};
   }
   return {prefix, need, cnt};
 }
