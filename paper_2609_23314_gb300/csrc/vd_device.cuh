@@ -133,6 +133,24 @@ __device__ __forceinline__ unsigned long long ld_shared_b64(uint32_t addr) {
   return r;
 }
 
+__device__ __forceinline__ void st_shared16(uint32_t addr, const uint4& v) {
+  asm volatile("st.shared.v4.u32 [%0], {%1,%2,%3,%4};" ::"r"(addr), "r"(v.x), "r"(v.y), "r"(v.z),
+               "r"(v.w)
+               : "memory");
+}
+
+__device__ __forceinline__ float ld_shared_f32(uint32_t addr) {
+  float r;
+  asm volatile("ld.shared.f32 %0, [%1];" : "=f"(r) : "r"(addr) : "memory");
+  return r;
+}
+
+__device__ __forceinline__ double ld_shared_f64(uint32_t addr) {
+  double r;
+  asm volatile("ld.shared.f64 %0, [%1];" : "=d"(r) : "r"(addr) : "memory");
+  return r;
+}
+
 __device__ __forceinline__ void st_cluster_u16(uint32_t addr, uint16_t v) {
   asm volatile("st.shared::cluster.u16 [%0], %1;" ::"r"(addr), "h"(v) : "memory");
 }

@@ -86,6 +86,13 @@ namespace vd {
 #ifndef VD_BLOCK_MIN_CTAS
 #define VD_BLOCK_MIN_CTAS 4
 #endif
+// Hole-fill block eviction: its one-CTA-per-unit launches hold the unit's
+// keys and slot list, which at prefill sizes already limit it to 3 CTAs per
+// SM, so it takes the registers of 3 (85 per thread): room for the
+// double-float retirement sums in its move stream.
+#ifndef VD_HF_BLOCK_MIN_CTAS
+#define VD_HF_BLOCK_MIN_CTAS 3
+#endif
 #ifndef VD_DECODE_MIN_CTAS
 #define VD_DECODE_MIN_CTAS 4
 #endif
@@ -1115,6 +1122,133 @@ __device__ __forceinline__ void move_rows_ring(uint16_t* kb, uint16_t* vb, int d
   cp_async_wait<0>();
 }
 
+// Hole-fill block events: the kept rows at or above N move into the evicted
+// slots below N, and, with the running mean, the evicted rows leave the
+// running sum in the same stream.  ev_of(i), i < ne = n - N, lists the
+// evicted rows ascending: the first h are the holes below N, which receive
+// the movers src_of(i); the rest lie at or above N and are only subtracted.
+// Threads keep one 16-byte column chunk of [K | V] (compact_slice's
+// mapping), so each thread reads a hole's old bytes and writes the mover's
+// into it itself, after both copies have landed, and no barrier is needed
+// between ring stages; sources and holes never overlap.  Thread chunks in the
+// scored tensor ([sc_lo, sc_hi) of [K | V], when `retire`) accumulate minus
+// the evicted rows in double-float; the partials are added per column in a
+// fixed order and base[c] plus them is written to rsum_out[c] for this CTA's
+// columns of the scored tensor (tchunk0, tchunks).  Rows at or above
+// first_stage are read from the staging buffers kn / vn.  A row outside
+// [0, n) is skipped and recorded as kStInternal.
+template <class Ring, bool PACKED, class SrcOf, class EvOf>
+__device__ __forceinline__ void move_rows_retire(uint16_t* kb, uint16_t* vb, int d, int chunk0,
+                                                 int cps, int h, int ne, int n, SrcOf src_of,
+                                                 EvOf ev_of, unsigned* status, const uint16_t* kn,
+                                                 const uint16_t* vn, int first_stage,
+                                                 uint32_t ring, bool retire, int sc_lo,
+                                                 int sc_hi, int tchunk0, int tchunks,
+                                                 uint32_t base, double* rsum_out) {
+  static_assert(Ring::kItems >= 2, "one ring slot for the mover, one for the evicted row");
+  constexpr int kStages = Ring::kStages;
+  const int tid = threadIdx.x, d8 = d >> 3;
+  const int rs = kThreads / cps;
+  const bool on = tid < rs * cps;
+  const int my_ch = chunk0 + tid % cps, my_off = tid / cps;
+  const bool scored = retire && on && my_ch >= sc_lo && my_ch < sc_hi;
+  uint16_t* col = my_ch < d8 ? kb + my_ch * 8 : vb + (my_ch - d8) * 8;
+  const uint16_t* scol = my_ch < d8 ? kn + my_ch * 8 : vn + (my_ch - d8) * 8;
+  auto rowp = [&](int r) -> const uint16_t* {
+    return r >= first_stage ? scol + (size_t)(r - first_stage) * d : col + (size_t)r * d;
+  };
+  // this thread's rows: my_off, my_off + rs, ... below h (moves) or ne (retired)
+  const int lim = scored ? ne : h;
+  const int cnt = on && lim > my_off ? (lim - my_off + rs - 1) / rs : 0;
+  const uint32_t my = ring + (uint32_t)tid * 16u;
+  auto slot = [&](int st, int k) { return my + (uint32_t)((st * Ring::kItems + k) * kThreads * 16); };
+  auto issue = [&](int j) {
+    if (j < cnt) {
+      const int i = my_off + j * rs;
+      const int ev = ev_of(i);
+      if ((unsigned)ev < (unsigned)n) {
+        if (i < h) {
+          const int sr = src_of(i);
+          if ((unsigned)sr < (unsigned)n) cp_async16(slot(j % kStages, 0), rowp(sr));
+          else record_status(status, kStInternal);
+        }
+        if (scored) cp_async16(slot(j % kStages, 1), rowp(ev));
+      } else {
+        record_status(status, kStInternal);
+      }
+    }
+    cp_async_commit();
+  };
+  float hi[8], lo[8];
+  unsigned long long hi2[4], lo2[4];
+#pragma unroll
+  for (int k = 0; k < 8; ++k) hi[k] = lo[k] = 0.f;
+#pragma unroll
+  for (int k = 0; k < 4; ++k) hi2[k] = lo2[k] = 0ull;
+  for (int j = 0; j < kStages; ++j) issue(j);
+  for (int j = 0; j < cnt; ++j) {
+    cp_async_wait<kStages - 1>();
+    const int i = my_off + j * rs;
+    const int ev = ev_of(i);
+    if ((unsigned)ev < (unsigned)n) {
+      if (scored) {  // minus the evicted row: its sign bits flipped (exact)
+        const uint4 q = ld_shared16(slot(j % kStages, 1));
+        const uint32_t w[4] = {q.x ^ 0x80008000u, q.y ^ 0x80008000u, q.z ^ 0x80008000u,
+                               q.w ^ 0x80008000u};
+        if constexpr (PACKED) {
+#pragma unroll
+          for (int k = 0; k < 4; ++k) ff2_accumulate(hi2[k], lo2[k], bf16x2_to_f2(w[k]));
+        } else {
+          float x[8];
+          unpack8(uint4{w[0], w[1], w[2], w[3]}, x);
+#pragma unroll
+          for (int k = 0; k < 8; ++k) ff_accumulate(hi[k], lo[k], x[k]);
+        }
+      }
+      if (i < h && (unsigned)src_of(i) < (unsigned)n)
+        st16(col + (size_t)ev * d, ld_shared16(slot(j % kStages, 0)));
+    }
+    issue(j + kStages);
+  }
+  cp_async_wait<0>();
+  if (!retire) return;
+  if constexpr (PACKED) {
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      f2_unpack(hi2[k], hi[2 * k], hi[2 * k + 1]);
+      f2_unpack(lo2[k], lo[2 * k], lo[2 * k + 1]);
+    }
+  }
+  // per-column partials of the rs threads that share a chunk (in the ring,
+  // free once every copy has landed: hi parts, then lo parts, 4 bytes per
+  // column), then their sum in the order of the threads
+  __syncthreads();
+  const uint32_t w = (uint32_t)cps * 32u;  // bytes of one thread row of partials
+  const uint32_t lo_off = (uint32_t)rs * w;
+  if (scored) {
+    const uint32_t at = ring + (uint32_t)my_off * w + (uint32_t)(my_ch - chunk0) * 32u;
+    st_shared16(at, uint4{__float_as_uint(hi[0]), __float_as_uint(hi[1]), __float_as_uint(hi[2]),
+                          __float_as_uint(hi[3])});
+    st_shared16(at + 16u, uint4{__float_as_uint(hi[4]), __float_as_uint(hi[5]),
+                                __float_as_uint(hi[6]), __float_as_uint(hi[7])});
+    st_shared16(at + lo_off, uint4{__float_as_uint(lo[0]), __float_as_uint(lo[1]),
+                                   __float_as_uint(lo[2]), __float_as_uint(lo[3])});
+    st_shared16(at + lo_off + 16u, uint4{__float_as_uint(lo[4]), __float_as_uint(lo[5]),
+                                         __float_as_uint(lo[6]), __float_as_uint(lo[7])});
+  }
+  __syncthreads();
+  if (tid < tchunks * 8) {
+    const int c = tchunk0 * 8 + tid;           // column of the scored tensor
+    const int lc = c + sc_lo * 8 - chunk0 * 8;  // its column within this CTA's slice
+    ff t{0.f, 0.f};
+    for (int o = 0; o < rs; ++o) {
+      const uint32_t at = ring + (uint32_t)o * w + (uint32_t)lc * 4u;
+      t = ff_add(t, ff{ld_shared_f32(at), ld_shared_f32(at + lo_off)});
+    }
+    rsum_out[c] = ld_shared_f64(base + (uint32_t)c * 8u) + (double)t.hi + (double)t.lo;
+  }
+}
+
 // VAR: 0 L2, 1 Dir, 2 Norm.  DECODE: one-token eviction (arg-min) instead of
 // the radix select.  HF: hole-fill layout (compiled separately, so the ordered
 // layout carries none of its code).  FUSED: the new rows are read from the
@@ -1592,14 +1726,19 @@ __device__ __forceinline__ void evict_unit(const EvictArgs& a) {
   // the scored tensor).  The appended rows were already summed for the mean
   // (all but Norm: S plus them is in S.snew); only the evicted rows are read
   // again.  Norm loads S before the row sum, whose latency hides it.
-  if (a.mu_running && tchunks > 0) {
+  // Hole-fill block events retire the evicted rows in the move stream
+  // (move_rows_retire) instead: here Norm only adds the appended rows, into
+  // S.snew, the base the move stream subtracts from.
+  constexpr bool kRetire = HF && !DECODE;
+  if (a.mu_running && tchunks > 0 && !(kRetire && VAR != 2)) {
     const int B = VAR != 2 ? 0 : a.B;
+    const int ne = kRetire ? 0 : n - Nb;
     double base = 0.0;
     if (tid < tchunks * 8) {
       const int c = tchunk0 * 8 + tid;
       base = VAR != 2 ? S.snew[c] : a.running_sum[(size_t)u * d + c] + 0.0;
     }
-    sum_rows<Ring, kPackedSum>(tchunk0, tchunks, tp, B + (n - Nb),
+    sum_rows<Ring, kPackedSum>(tchunk0, tchunks, tp, B + ne,
              [&](int i) {
                const int r =
                    i < B ? first_new + i : (DECODE ? e_first : (int)perm[Nb + (i - B)]);
@@ -1610,7 +1749,9 @@ __device__ __forceinline__ void evict_unit(const EvictArgs& a) {
              [&](int i) { return i < B ? 1.f : -1.f; }, S, ring);
     if (tid < tchunks * 8) {
       const int c = tchunk0 * 8 + tid;
-      a.running_sum[(size_t)u * d + c] = base + (double)S.acc_hi[c] + (double)S.acc_lo[c];
+      const double v = base + (double)S.acc_hi[c] + (double)S.acc_lo[c];
+      if (kRetire) S.snew[c] = v;
+      else a.running_sum[(size_t)u * d + c] = v;
     }
   }
 
@@ -1649,11 +1790,16 @@ __device__ __forceinline__ void evict_unit(const EvictArgs& a) {
       copy_new_rows(kb, vb, knu, vnu, d, chunk0, cps, first_stage, Nb - first_stage);
       __syncthreads();
     }
-    if constexpr (DECODE)
+    if constexpr (DECODE) {
       move_rows(kb, vb, d, chunk0, cps, h, n, src, dst, a.status, knu, vnu, first_stage);
-    else
-      move_rows_ring<Ring>(kb, vb, d, chunk0, cps, h, n, src, dst, a.status, knu, vnu,
-                           first_stage, ring);
+    } else {
+      // the scored tensor's chunks of [K | V]: K's [0, d8) or V's [d8, 2 d8)
+      const int sc_lo = a.score_k ? 0 : d8;
+      move_rows_retire<Ring, kPackedSum>(
+          kb, vb, d, chunk0, cps, h, n - Nb, n, src, dst, a.status, knu, vnu, first_stage, ring,
+          a.mu_running && tchunks > 0, sc_lo, sc_lo + d8, tchunk0, tchunks, smem_addr(S.snew),
+          a.running_sum + (size_t)u * d);
+    }
     if (rank == 0) {
       for (int r = max(first_new, 0) + tid; r < Nb; r += kThreads) posu[r] = pnew + (r - first_new);
       int32_t* ko = a.kept_out ? a.kept_out + (size_t)u * a.N : nullptr;
@@ -1683,6 +1829,7 @@ __device__ __forceinline__ void evict_unit(const EvictArgs& a) {
 template <int VAR, bool DECODE, bool HF, bool FUSED, bool SCORE = false>
 __global__ void __launch_bounds__(kThreads, SCORE    ? VD_SCORE_MIN_CTAS
                                             : DECODE ? VD_DECODE_MIN_CTAS
+                                            : HF     ? VD_HF_BLOCK_MIN_CTAS
                                                      : VD_BLOCK_MIN_CTAS)
     evict_kernel(const EvictArgs a) {
   grid_launch_dependents();
