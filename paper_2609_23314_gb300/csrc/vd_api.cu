@@ -71,8 +71,12 @@ __global__ void vd_len_add_kernel(int32_t* len, int n_seq, int cap, int B) {
 
 // Mirrors the eviction kernel's per-sequence decision exactly.  added: the
 // rows a fused append adds to len (0 when they were appended beforehand).
+// Launched as a programmatic dependent of the eviction (which lets its
+// dependents be scheduled at once): it is resident before the eviction ends
+// and waits for it to complete before reading or writing len.
 __global__ void vd_len_clamp_kernel(int32_t* len, const int32_t* N_dev, int N, int n_seq,
                                     int cap, int B, int running, int decode, int added) {
+  vd::grid_dependency_wait();
   const int s = blockIdx.x * blockDim.x + threadIdx.x;
   if (s >= n_seq) return;
   const int n0 = len[s];
@@ -626,11 +630,21 @@ vd_status run(const vd_cache* c, int32_t N, const int32_t* N_dev, int32_t B, vd_
     r = launch(kern, units, a.cluster, smem, &a, s);
   }
   if (r != VD_OK || score_only) return r;
-  const int threads = 256;
-  vd_len_clamp_kernel<<<(c->n_seq + threads - 1) / threads, threads, 0, s>>>(
-      c->len, N_dev, N, c->n_seq, c->capacity, a.B, a.mu_running, decode ? 1 : 0,
-      fused ? a.B : 0);
-  if (cudaGetLastError() != cudaSuccess) return VD_ERR_CUDA;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)((c->n_seq + kThreads - 1) / kThreads));
+  cfg.blockDim = dim3(kThreads);
+  cfg.stream = s;
+  cudaLaunchAttribute pdl;
+  pdl.id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  pdl.val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = &pdl;
+  cfg.numAttrs = 1;
+  if (cudaLaunchKernelEx(&cfg, vd_len_clamp_kernel, c->len, N_dev, N, c->n_seq, c->capacity,
+                         (int)a.B, (int)a.mu_running, decode ? 1 : 0, fused ? (int)a.B : 0) !=
+      cudaSuccess) {
+    cudaGetLastError();
+    return VD_ERR_CUDA;
+  }
   return VD_OK;
 }
 
