@@ -713,7 +713,8 @@ struct Selection {
 };
 
 // first_ready: S.hist[0] already holds this CTA's counts of the keys' top
-// byte (built by the score pass), so the first pass skips its counting loop.
+// byte (built by the score pass), so the first pass skips its counting loop,
+// and S.hist[1] was zeroed with it, so the second pass does not zero it.
 //
 // As soon as a pass leaves at most kThreads keys in the cluster that share
 // the threshold's prefix (the candidates), the remaining passes are replaced
@@ -733,7 +734,7 @@ __device__ __forceinline__ Selection cluster_radix_select(KeyOf key_of, int R, i
     const int shift = 24 - 8 * pass;
     uint32_t* h = S.hist[pass & 1];
     const bool counted = pass == 0 && first_ready;
-    if (!counted) {
+    if (!(first_ready && pass <= 1)) {
       h[tid] = 0;
       __syncthreads();
     }
@@ -743,11 +744,16 @@ __device__ __forceinline__ Selection cluster_radix_select(KeyOf key_of, int R, i
       uint32_t key = 0u;
       if (j < R) key = key_of(j, ok);
       const bool match = ok && (key & pmask) == prefix;
-      const unsigned act = __ballot_sync(kFull, match);
-      if (match) {
-        const uint32_t dig = (key >> shift) & 255u;
-        const unsigned peers = __match_any_sync(act, dig);
-        if (lane == __ffs(peers) - 1) atomicAdd(&h[dig], (uint32_t)__popc(peers));
+      const uint32_t dig = (key >> shift) & 255u;
+      if (pass == 0) {
+        // the top bytes of nearby scores coincide: one atomic per distinct digit
+        const unsigned act = __ballot_sync(kFull, match);
+        if (match) {
+          const unsigned peers = __match_any_sync(act, dig);
+          if (lane == __ffs(peers) - 1) atomicAdd(&h[dig], (uint32_t)__popc(peers));
+        }
+      } else if (match) {
+        atomicAdd(&h[dig], 1u);  // later digits are spread: plain shared atomics
       }
     }
     if (C > 1) cluster_sync(); else __syncthreads();
@@ -1372,6 +1378,7 @@ __device__ __forceinline__ void evict_unit(const EvictArgs& a) {
   const bool hist_pre = !DECODE && !score_only && a.weights == nullptr;
   if (hist_pre) {
     S.hist[0][tid] = 0;
+    S.hist[1][tid] = 0;  // the select's second pass counts into it without zeroing
     __syncthreads();
   }
   // ---- 1. mean ---------------------------------------------------------
