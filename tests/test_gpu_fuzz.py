@@ -3,7 +3,8 @@
 Each case draws a shape (sequences, layers, KV heads, a head dim that is a
 multiple of 8 up to 256), a budget N, a block size B (1 for decode), ragged
 lengths at or below N, a scoring rule, a mean mode, a layout and a cluster
-size, per-sequence budgets or not, fills the cache from the workload
+size (with it, in 40 % of the cases, a split launch: the first units one
+CTA each, the rest on clusters of that size), per-sequence budgets or not, fills the cache from the workload
 generators, and runs two events through vd_append_evict_block /
 vd_append_evict_decode (or, in some cases, the two-call form: vd_append,
 then the eviction of that layout).  Every unit of every
@@ -59,7 +60,18 @@ def draw_case(i, medium=False):
                 var=int(r.integers(0, 3)), mu=int(r.integers(0, 2)),
                 holefill=bool(r.random() < 0.4),
                 cluster=int(r.choice(allowed)) if r.random() < 0.5 else 0,
-                gen=str(r.choice(["gauss_outlier", "student_t"])), seed=int(r.integers(1, 1 << 30)))
+                gen=str(r.choice(["gauss_outlier", "student_t"])), seed=int(r.integers(1, 1 << 30)),
+                split=float(r.random()))
+
+
+def force_split(c, monkeypatch):
+    """With a forced cluster size, 40 % of the cases also force a split
+    launch: the first s units (1 <= s < U) one CTA each, the rest on
+    clusters of the forced size."""
+    U = c["n_seq"] * c["L"] * c["H"]
+    if c["cluster"] and U >= 2 and c["split"] < 0.4:
+        s = 1 + min(U - 2, int(c["split"] / 0.4 * (U - 1)))
+        monkeypatch.setenv("VD_SOLO_UNITS", str(s))
 
 
 @pytest.mark.parametrize("case", [(i, False) for i in range(N_CASES)] +
@@ -70,6 +82,7 @@ def test_fused_random_shapes(orc, case, monkeypatch):
     c = draw_case(*case)
     if c["cluster"]:
         monkeypatch.setenv("VD_CLUSTER_SIZE", str(c["cluster"]))
+    force_split(c, monkeypatch)
     d, N, B, cap = c["d"], c["N"], c["B"], c["cap"]
     cache = new_cache(c["n_seq"], c["L"], c["H"], cap, d)
     U, us, per_seq = cache.units, cache.unit_shape(), c["L"] * c["H"]
@@ -164,7 +177,7 @@ def draw_ex(i):
                 mu=int(r.integers(0, 2)),
                 cluster=int(r.choice(allowed)) if r.random() < 0.5 else 0,
                 gen=str(r.choice(["gauss_outlier", "student_t"])), seed=int(r.integers(1, 1 << 30)),
-                fused=bool(r.random() < 0.5))
+                fused=bool(r.random() < 0.5), split=float(r.random()))
 
 
 @pytest.mark.parametrize("case", range(N_EX))
@@ -181,6 +194,7 @@ def test_ex_random_options(orc, case, monkeypatch):
     c = draw_ex(case)
     if c["cluster"]:
         monkeypatch.setenv("VD_CLUSTER_SIZE", str(c["cluster"]))
+    force_split(c, monkeypatch)
     d, N, B, cap, var = c["d"], c["N"], c["B"], c["cap"], c["var"]
     cache = new_cache(c["n_seq"], c["L"], c["H"], cap, d)
     U, us, per_seq = cache.units, cache.unit_shape(), c["L"] * c["H"]
