@@ -40,10 +40,16 @@
  *   relative to the score itself (a few 1e-7 in practice).  Ranking: a NaN
  *   score ranks below every number, +0 and -0 are equal.
  * - Launches: one eviction kernel per call, plus a one-thread-per-sequence
- *   length update.  A short cache (capacity <= 1024, 4 * capacity * head_dim
- *   <= 64 KB, at most 16 units per sequence, at most two units per SM) takes
- *   a kernel that keeps the unit in shared memory and updates the lengths
- *   itself: one launch in all.  Results follow the same rules either way.
+ *   length update (a programmatic dependent launch of the eviction, all on
+ *   `stream`).  A hole-fill block eviction or a score-only call that fits
+ *   one wave at one CTA per unit but has more units than the GPU has SMs
+ *   runs the eviction kernel as two launches over disjoint units, the second
+ *   a programmatic dependent of the first, so that no SM carries a whole
+ *   unit more than the others.  A short cache (capacity <= 1024,
+ *   4 * capacity * head_dim <= 64 KB, at most 16 units per sequence, at most
+ *   two units per SM) takes a kernel that keeps the unit in shared memory
+ *   and updates the lengths itself: one launch in all.  Results follow the
+ *   same rules either way, and every call can be captured in a CUDA graph.
  */
 #ifndef VD_H
 #define VD_H
@@ -139,7 +145,8 @@ vd_status vd_evict_block(const vd_cache* c, int32_t N, const int32_t* N_dev, int
                          int32_t* kept_idx_out, float* scores_out, vd_stream_t stream);
 
 /* One step of block prompt processing (Sec. 2.2, Eq. block_processing:
- * C_i = pi_N([C_{i-1} || block_i])) in a single launch: the same result as
+ * C_i = pi_N([C_{i-1} || block_i])) with the append fused into the
+ * eviction kernel: the same result as
  * vd_append(c, k_new, v_new, B) followed by vd_evict_block(c, N, N_dev, B,
  * var, mu, running_sum, kept_idx_out, scores_out) -- the same kept slots,
  * scores, compacted K/V bytes in slots [0, new len), running sum and len --
@@ -179,8 +186,8 @@ vd_status vd_evict_decode(const vd_cache* c, int32_t N, const int32_t* N_dev, vd
                           vd_mu_mode mu, double* running_sum, int32_t* evicted_out,
                           int32_t* kept_idx_out, float* scores_out, vd_stream_t stream);
 
-/* One decode step in one launch: the same result as vd_append(c, k_new,
- * v_new, 1) followed by vd_evict_decode (or, with pos and pos_first_new, by
+/* One decode step, the append fused into the eviction kernel: the same
+ * result as vd_append(c, k_new, v_new, 1) followed by vd_evict_decode (or, with pos and pos_first_new, by
  * vd_evict_decode_holefill), with the new token read straight from the
  * caller's buffers and written into the cache only if it survives.
  *   k_new, v_new  bf16 device [n_seq][n_layer][n_kv_head][1][head_dim],
@@ -241,7 +248,8 @@ vd_status vd_evict_block_ex(const vd_cache* c, int32_t N, const int32_t* N_dev, 
                             int32_t score_keys, const float* attn, int32_t* kept_idx_out,
                             float* scores_out, float* dispersion_out, vd_stream_t stream);
 
-/* vd_append followed by vd_evict_block_ex in one launch, as
+/* vd_append followed by vd_evict_block_ex with the append fused into the
+ * eviction kernel, as
  * vd_append_evict_block is for vd_evict_block (one step of Sec. 2.2,
  * Eq. block_processing, with the scoring options above): k_new, v_new are
  * bf16 device [n_seq][n_layer][n_kv_head][B][head_dim], 16-byte aligned,
