@@ -187,8 +187,9 @@ vd_status vd_evict_decode(const vd_cache* c, int32_t N, const int32_t* N_dev, vd
                           int32_t* kept_idx_out, float* scores_out, vd_stream_t stream);
 
 /* One decode step, the append fused into the eviction kernel: the same
- * result as vd_append(c, k_new, v_new, 1) followed by vd_evict_decode (or, with pos and pos_first_new, by
- * vd_evict_decode_holefill), with the new token read straight from the
+ * result as vd_append(c, k_new, v_new, 1) followed by vd_evict_decode (or,
+ * with pos and pos_first_new, by vd_evict_decode_holefill), with the new
+ * token read straight from the
  * caller's buffers and written into the cache only if it survives.
  *   k_new, v_new  bf16 device [n_seq][n_layer][n_kv_head][1][head_dim],
  *                 16-byte aligned, read only.
